@@ -1,0 +1,191 @@
+/*
+ * ffh.h -- C ABI of libffh, the FlipFlop Hessian estimator on one GB300 GPU.
+ *
+ * The estimator (Birnick & Saab, "WaterKron and FlipFlop Hessian", Section 5) fits a
+ * Kronecker-factored Hessian A (x) B, A in R^{n x n} (input side), B in R^{m x m}
+ * (output side), to the calibration samples of a linear layer W in R^{m x n}.  For
+ * rank-one samples G_k = g_k x_k^T (x_k in R^n the layer input, g_k in R^m the output
+ * gradient) the flip-flop updates are
+ *
+ *     B <- 1/(N n) sum_k (x_k^T A^-1 x_k) g_k g_k^T,
+ *     A <- 1/(N m) sum_k (g_k^T B^-1 g_k) x_k x_k^T,
+ *
+ * iterated from A_0 = I_n, one iteration = B-update then A-update (Appendix B).  The
+ * proportionality constants of Section 5 are fixed to the matrix-normal MLE values
+ * above; after every iteration A is rescaled to tr(A) = n and B by the inverse
+ * factor, which leaves A (x) B unchanged (the fixed point is unique only up to that
+ * scale).
+ *
+ * Conventions common to every call:
+ *  - Matrices are row-major.  X is N x n (row k = x_k^T), G is N x m (row k = g_k^T),
+ *    Gk is N x m x n (sample k is the m x n matrix G_k).  A is n x n, B is m x m, both
+ *    written in full symmetric storage, fp32.
+ *  - "device or host": a pointer may address device memory or host memory (pinned or
+ *    pageable).  Host inputs are copied into the handle's workspace and host outputs
+ *    copied back inside the call; device inputs are read in place.  All device memory
+ *    passed in is owned by the caller and must stay valid until the call returns.
+ *  - Every call enqueues its work on the handle's CUDA stream and synchronises that
+ *    stream once before returning (the status of the fit is read back then).
+ *  - A handle must not be used by two host threads at once.  Each handle owns a
+ *    workspace on the current device, grown on demand and freed by ffh_destroy.
+ *  - On error the outputs are undefined; ffh_last_error() describes the error.
+ */
+#ifndef FFH_H
+#define FFH_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct ffh_ctx* ffh_t;
+
+typedef enum {
+  FFH_OK = 0,
+  FFH_ERR_INVALID_ARG = 1, /* null pointer, bad size, misaligned row pitch, iters < 1 */
+  FFH_ERR_NOT_SPD = 2,     /* a Cholesky pivot was <= 0 or not finite */
+  FFH_ERR_RANK = 3,        /* N < max(n, m) without damping: the MLE need not exist */
+  FFH_ERR_OOM = 4,         /* workspace allocation failed */
+  FFH_ERR_CUDA = 5,        /* a CUDA runtime call failed */
+  FFH_ERR_TIMEOUT = 6,     /* a bounded device-side wait expired; the kernel returned */
+  FFH_ERR_UNSUPPORTED = 7  /* no sm_100-family GPU, or an option this build lacks */
+} ffh_status;
+
+typedef enum { FFH_BF16 = 0, FFH_F32 = 1 } ffh_dtype;
+
+/* Hessian variants of Table 1 that share the alternating loop. */
+typedef enum {
+  FFH_FLIPFLOP = 0,  /* A = E[(g^T B^-1 g) x x^T], B = E[(x^T A^-1 x) g g^T] (Section 5) */
+  FFH_FROBENIUS = 1  /* A = E[(g^T B g) x x^T]/||B||_F^2, B = E[(x^T A x) g g^T]/||A||_F^2 */
+} ffh_variant;
+
+/* Test-only fault injection codes (ffh_options.fault). */
+enum {
+  FFH_FAULT_NONE = 0,
+  FFH_FAULT_OOM = 1,          /* the next workspace allocation reports failure */
+  FFH_FAULT_BAD_PIVOT = 2,    /* the first Cholesky sees a NaN pivot -> FFH_ERR_NOT_SPD */
+  FFH_FAULT_LOST_COPY = 3     /* the Gram kernel drops one staged copy, so its consumer's
+                                 bounded wait expires -> FFH_ERR_TIMEOUT (device context
+                                 stays usable) */
+};
+
+/* Zero-initialised options are the defaults. */
+typedef struct {
+  int32_t dtype;           /* ffh_dtype of X and G (Gk is always fp32) */
+  float damping;           /* lambda >= 0: F <- F + lambda * mean(diag F) * I right after
+                              each update, the mean taken before the shift (Appendix B
+                              uses 0.1; default 0) */
+  int32_t variant;         /* ffh_variant */
+  const float* init_A;     /* optional warm start (n x n fp32, SPD, device or host);
+                              NULL: A_0 = I_n (Appendix B) */
+  int32_t final_loglik;    /* 1: also evaluate the log-likelihood at the returned (A, B)
+                              (one more Cholesky and quadratic-form pass) */
+  int32_t kernel;          /* 0: tensor-core kernels (tcgen05); 1: CUDA-core kernels
+                              (slower; for cross-checking the tensor-core path) */
+  int32_t fault;           /* FFH_FAULT_* (tests only) */
+  int32_t profile;         /* 1: time the Gram, quadratic-form and Cholesky kernels with
+                              CUDA events on the handle's stream (see ffh_get_timings) */
+  int32_t reserved[4];     /* must be zero */
+} ffh_options;
+
+/* Kernel timings accumulated over the calls made with opt.profile = 1. */
+typedef struct {
+  double gram_ms;          /* total device time of the weighted-Gram main kernel */
+  int64_t gram_launches;
+  double qform_ms;         /* total device time of the quadratic-form kernel */
+  int64_t qform_launches;
+  double chol_ms;          /* total device time of Cholesky + inverse (all their kernels) */
+  int64_t chol_calls;
+  int64_t kernel_launches; /* every kernel libffh launched in this process (profile or not) */
+} ffh_timings;
+
+/* Library version as major*10000 + minor*100 + patch. */
+int32_t ffh_version(void);
+
+/* Create a handle bound to the current CUDA device and to `cuda_stream` (a
+ * cudaStream_t; NULL = the legacy default stream).  `opt` may be NULL (defaults).
+ * Fails with FFH_ERR_UNSUPPORTED unless the device is compute capability 10.x. */
+ffh_status ffh_create(ffh_t* out, const ffh_options* opt, void* cuda_stream);
+
+/* Replace the options / the stream of an existing handle. */
+ffh_status ffh_set_options(ffh_t h, const ffh_options* opt);
+ffh_status ffh_set_stream(ffh_t h, void* cuda_stream);
+
+/* Free the workspace and the handle.  NULL is accepted. */
+ffh_status ffh_destroy(ffh_t h);
+
+/* Human-readable description of the last error on this handle ("" if none).  The
+ * string is owned by the handle and valid until its next call. */
+const char* ffh_last_error(ffh_t h);
+
+/* FlipFlop fit to rank-one samples (Section 5 updates, Appendix B settings).
+ *   X      N x n, row pitch n elements, dtype opt.dtype (device or host)
+ *   G      N x m, row pitch m elements, same dtype
+ *   iters  maximum number of iterations (>= 1); one iteration = B-update, A-update
+ *   tol    stop after iteration t when delta_t < tol, where
+ *          delta_t = max_{F in {A,B}} ||F_t/tr F_t - F_{t-1}/tr F_{t-1}||_F / ||F_t/tr F_t||_F
+ *          (delta_1 = +inf); tol = 0 runs exactly `iters` iterations
+ *   A_out  n x n fp32 (device or host): A with tr(A) = n
+ *   B_out  m x m fp32 (device or host)
+ * bf16 rows must be 16-byte aligned: n and m multiples of 8 for FFH_BF16 (fp32 inputs
+ * accept any n, m).  Reaching `iters` without meeting `tol` is not an error; see
+ * ffh_get_stats.  Errors: INVALID_ARG, RANK, NOT_SPD, OOM, CUDA, TIMEOUT. */
+ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, int64_t n, int64_t m,
+                   int32_t iters, float tol, float* A_out, float* B_out);
+
+/* FlipFlop fit to general matrix samples G_k in R^{m x n} (Section 5, the first form of
+ * each update):  B <- 1/(N n) sum_k G_k A^-1 G_k^T,  A <- 1/(N m) sum_k G_k^T B^-1 G_k.
+ *   Gk  N x m x n fp32, row-major per sample (device or host).
+ * Other arguments, normalisation and errors as ffh_fit.  n and m multiples of 4. */
+ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_t n, int64_t m,
+                          int32_t iters, float tol, float* A_out, float* B_out);
+
+/* Statistics of the last fit on this handle (host pointers, each nullable).
+ *   iters_done    iterations run
+ *   delta         delta of the last iteration (+inf after one iteration)
+ *   loglik_trace  receives up to `capacity` values: the Gaussian log-likelihood
+ *                 -1/2 [N m log|A| + N n log|B| + sum_k tr(B^-1 G_k A^-1 G_k^T)]
+ *                 after every half-step: l(A_0,B_1), l(A_1,B_1), l(A_1,B_2), ...;
+ *                 the last entry is NaN unless opt.final_loglik was set
+ *   mean_qr       receives up to `capacity` values of mean_k q_k r_k after every
+ *                 half-step (m n for an undamped fit: the trace identity)
+ * Returns the number of trace entries available (2 * iters_done) via *n_trace. */
+ffh_status ffh_get_stats(ffh_t h, int32_t* iters_done, double* delta, double* loglik_trace,
+                         double* mean_qr, int32_t capacity, int32_t* n_trace);
+
+/* Copy the accumulated timings into *out; reset = 1 clears them afterwards (the
+ * process-wide launch counter is not reset). */
+ffh_status ffh_get_timings(ffh_t h, ffh_timings* out, int32_t reset);
+
+/* ---- single steps of the fit (device pointers only; on the handle's stream) ---- */
+
+/* Weighted Gram (the E[w v v^T] of the Section 5 updates; w = NULL gives the plain
+ * Gram E[v v^T] of Table 1's Input / Marginal Hessians):
+ *   C = scale * sum_k w_k v_k v_k^T = scale * V^T diag(w) V
+ *   V      N x d, row pitch d, dtype opt.dtype (bf16: d multiple of 8)
+ *   w      N fp32 weights, or NULL for w = 1
+ *   C_out  d x d fp32, full symmetric storage (lower triangle computed, mirrored). */
+ffh_status ffh_weighted_gram(ffh_t h, const void* V, const float* w, int64_t N, int64_t d,
+                             float scale, float* C_out);
+
+/* Quadratic forms with an inverse Cholesky factor (the weights x^T A^-1 x of Section 5):
+ *   q_k = ||Linv v_k||^2 = v_k^T F^-1 v_k  when Linv = L^-1, L L^T = F
+ *   V      N x d (dtype opt.dtype), Linv d x d fp32 lower-triangular, q_out N fp32. */
+ffh_status ffh_quad_form(ffh_t h, const void* V, const float* Linv, int64_t N, int64_t d,
+                         float* q_out);
+
+/* Cholesky factor and its inverse (Section 2 notation: L lower, L L^T = F, L_ii > 0):
+ *   F        d x d fp32 symmetric (lower triangle read)
+ *   L_out    d x d fp32, lower triangle (upper set to 0); nullable
+ *   Linv_out d x d fp32, L^-1 (lower, upper 0); nullable
+ *   logdet   host double, log|F| = 2 sum_i log L_ii; nullable
+ * Errors: NOT_SPD if a pivot is <= 0 or not finite. */
+ffh_status ffh_cholesky(ffh_t h, const float* F, int64_t d, float* L_out, float* Linv_out,
+                        double* logdet);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FFH_H */

@@ -1,0 +1,746 @@
+// libffh C ABI: handle, workspace, and the host-side driver of the FlipFlop fit.
+//
+// One fit enqueues, per iteration t (Section 5 updates, Appendix B order):
+//   [t = 1, A_0 = I]  q_k = ||x_k||^2
+//   [otherwise]       L = chol(A_{t-1}), M = L^-1 (bf16 copy), q_k = ||M x_k||^2
+//   B_t = 1/(N n) G^T diag(q) G   (+ damping)
+//   L = chol(B_t), M = L^-1,        r_k = ||M g_k||^2
+//   A_t = 1/(N m) X^T diag(r) X   (+ damping)
+//   s = tr(A_t)/n;  A_t /= s;  B_t *= s
+//   convergence statistics of A_t, B_t against A_{t-1}, B_{t-1}
+// all on the handle's stream; the host reads the device status once at the end (and
+// once per iteration only when tol > 0).
+#include <stdarg.h>
+
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "ffh_internal.cuh"
+
+namespace ffh {
+cudaError_t launch_lower_to_bf16(const float* src, int64_t d, int64_t lds, __nv_bfloat16* dst,
+                                 int64_t ldd, cudaStream_t s);
+cudaError_t launch_trace(const float* F, int64_t d, double* out, cudaStream_t s);
+}  // namespace ffh
+
+using namespace ffh;
+
+struct ffh_ctx {
+  ffh_options opt{};
+  cudaStream_t stream = nullptr;
+  int device = 0;
+  std::string err;
+  void* ws = nullptr;
+  size_t ws_bytes = 0;
+  // last fit
+  int iters_done = 0;
+  int64_t N = 0, n = 0, m = 0;
+  bool final_loglik = false;
+  std::vector<IterRecord> recs;  // index 1..iters_done
+  // profiling (opt.profile): CUDA events recorded around the timed kernels
+  double prof_ms[3] = {0, 0, 0};        // gram, qform, cholesky
+  long long prof_n[3] = {0, 0, 0};
+  std::vector<cudaEvent_t> ev_pool;
+  size_t ev_used = 0;
+  struct Pending {
+    int kind;
+    cudaEvent_t a, b;
+  };
+  std::vector<Pending> pending;
+};
+
+namespace {
+
+struct Carve {
+  char* base;
+  size_t off = 0;
+  explicit Carve(void* b) : base(static_cast<char*>(b)) {}
+  template <class T>
+  T* take(size_t count, size_t align = 256) {
+    off = (off + align - 1) & ~(align - 1);
+    T* p = base ? reinterpret_cast<T*>(base + off) : nullptr;
+    off += count * sizeof(T);
+    return p;
+  }
+};
+
+ffh_status fail(ffh_t h, ffh_status st, const char* fmt, ...) {
+  if (h) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    h->err = buf;
+  }
+  return st;
+}
+
+#define CK(call)                                                                        \
+  do {                                                                                  \
+    cudaError_t e_ = (call);                                                            \
+    if (e_ != cudaSuccess)                                                              \
+      return fail(h, FFH_ERR_CUDA, "%s failed: %s (%s:%d)", #call, cudaGetErrorString(e_), \
+                  __FILE__, __LINE__);                                                  \
+  } while (0)
+
+bool is_device_ptr(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
+int64_t pad8(int64_t d) { return (d + 7) / 8 * 8; }
+
+ffh_status ensure_ws(ffh_t h, size_t bytes) {
+  if (h->opt.fault == FFH_FAULT_OOM) return fail(h, FFH_ERR_OOM, "workspace allocation failed (injected)");
+  if (bytes <= h->ws_bytes && h->ws) return FFH_OK;
+  CK(cudaStreamSynchronize(h->stream));
+  if (h->ws) {
+    cudaFree(h->ws);
+    h->ws = nullptr;
+    h->ws_bytes = 0;
+  }
+  void* p = nullptr;
+  if (cudaMalloc(&p, bytes) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(h, FFH_ERR_OOM, "workspace allocation of %zu bytes failed", bytes);
+  }
+  h->ws = p;
+  h->ws_bytes = bytes;
+  return FFH_OK;
+}
+
+enum { PROF_GRAM = 0, PROF_QFORM = 1, PROF_CHOL = 2 };
+
+cudaEvent_t next_event(ffh_t h) {
+  if (h->ev_used == h->ev_pool.size()) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    h->ev_pool.push_back(e);
+  }
+  return h->ev_pool[h->ev_used++];
+}
+
+// Start a timed region of `kind` on the handle's stream (no-op unless opt.profile).
+cudaEvent_t prof_begin(ffh_t h) {
+  if (!h->opt.profile) return nullptr;
+  cudaEvent_t e = next_event(h);
+  if (e) cudaEventRecord(e, h->stream);
+  return e;
+}
+
+void prof_end(ffh_t h, int kind, cudaEvent_t a, cudaEvent_t b_recorded = nullptr) {
+  if (!a) return;
+  cudaEvent_t b = b_recorded;
+  if (!b) {
+    b = next_event(h);
+    if (!b) return;
+    cudaEventRecord(b, h->stream);
+  }
+  h->pending.push_back({kind, a, b});
+}
+
+// After a stream synchronisation: fold the recorded intervals into the totals.
+void prof_resolve(ffh_t h) {
+  for (auto& p : h->pending) {
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, p.a, p.b) == cudaSuccess) {
+      h->prof_ms[p.kind] += ms;
+      h->prof_n[p.kind] += 1;
+    } else {
+      cudaGetLastError();
+    }
+  }
+  h->pending.clear();
+  h->ev_used = 0;
+}
+
+ffh_status read_status(ffh_t h, DevStatus* st_dev) {
+  DevStatus st;
+  CK(cudaMemcpyAsync(&st, st_dev, sizeof(st), cudaMemcpyDeviceToHost, h->stream));
+  CK(cudaStreamSynchronize(h->stream));
+  prof_resolve(h);
+  if (st.error == FFH_ERR_NOT_SPD)
+    return fail(h, FFH_ERR_NOT_SPD, "Cholesky pivot <= 0 or not finite at index %d", st.error_info);
+  if (st.error == FFH_ERR_TIMEOUT)
+    return fail(h, FFH_ERR_TIMEOUT, "bounded device wait expired (site %d)", st.error_info);
+  if (st.error) return fail(h, (ffh_status)st.error, "device error %d (info %d)", st.error, st.error_info);
+  return FFH_OK;
+}
+
+// Input staging: a device bf16 view of V (for the tensor-core kernels) and a device
+// view in the caller's dtype (for the CUDA-core kernels).
+struct Staged {
+  const __nv_bfloat16* bf = nullptr;
+  int64_t ld_bf = 0;
+  const void* raw = nullptr;
+  int64_t ld_raw = 0;
+};
+
+struct GramTables {
+  GramPlan plan{};
+  int2* tiles = nullptr;
+  int* lut = nullptr;
+};
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+extern "C" {
+
+int32_t ffh_version(void) { return 100; }
+
+ffh_status ffh_create(ffh_t* out, const ffh_options* opt, void* cuda_stream) {
+  if (!out) return FFH_ERR_INVALID_ARG;
+  *out = nullptr;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return FFH_ERR_CUDA;
+  }
+  int major = 0;
+  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+  if (major != 10) return FFH_ERR_UNSUPPORTED;
+  ffh_ctx* h = new ffh_ctx();
+  if (opt) h->opt = *opt;
+  h->stream = static_cast<cudaStream_t>(cuda_stream);
+  h->device = dev;
+  *out = h;
+  return FFH_OK;
+}
+
+ffh_status ffh_set_options(ffh_t h, const ffh_options* opt) {
+  if (!h) return FFH_ERR_INVALID_ARG;
+  h->opt = opt ? *opt : ffh_options{};
+  return FFH_OK;
+}
+
+ffh_status ffh_set_stream(ffh_t h, void* cuda_stream) {
+  if (!h) return FFH_ERR_INVALID_ARG;
+  h->stream = static_cast<cudaStream_t>(cuda_stream);
+  return FFH_OK;
+}
+
+ffh_status ffh_destroy(ffh_t h) {
+  if (!h) return FFH_OK;
+  if (h->ws) {
+    cudaStreamSynchronize(h->stream);
+    cudaFree(h->ws);
+  }
+  for (cudaEvent_t e : h->ev_pool) cudaEventDestroy(e);
+  delete h;
+  return FFH_OK;
+}
+
+const char* ffh_last_error(ffh_t h) { return h ? h->err.c_str() : "null handle"; }
+
+}  // extern "C"
+
+// ---------------------------------------------------------------------------
+namespace {
+
+ffh_status validate_opt(ffh_t h) {
+  const ffh_options& o = h->opt;
+  if (o.dtype != FFH_BF16 && o.dtype != FFH_F32) return fail(h, FFH_ERR_INVALID_ARG, "bad dtype %d", o.dtype);
+  if (!(o.damping >= 0.f) || !std::isfinite(o.damping))
+    return fail(h, FFH_ERR_INVALID_ARG, "damping must be finite and >= 0");
+  if (o.variant != FFH_FLIPFLOP && o.variant != FFH_FROBENIUS)
+    return fail(h, FFH_ERR_INVALID_ARG, "bad variant %d", o.variant);
+  if (o.kernel != 0 && o.kernel != 1) return fail(h, FFH_ERR_INVALID_ARG, "bad kernel %d", o.kernel);
+  return FFH_OK;
+}
+
+// Stage one sample matrix (N x d, caller dtype): returns device views.
+ffh_status stage_input(ffh_t h, const void* V, bool on_dev, int64_t N, int64_t d,
+                       __nv_bfloat16* bf_buf, float* f32_stage, Staged* out) {
+  const int dtype = h->opt.dtype;
+  if (dtype == FFH_BF16) {
+    if (on_dev) {
+      out->bf = static_cast<const __nv_bfloat16*>(V);
+    } else {
+      CK(cudaMemcpyAsync(bf_buf, V, (size_t)N * d * 2, cudaMemcpyHostToDevice, h->stream));
+      out->bf = bf_buf;
+    }
+    out->ld_bf = d;
+    out->raw = out->bf;
+    out->ld_raw = d;
+    return FFH_OK;
+  }
+  const float* src = static_cast<const float*>(V);
+  if (!on_dev) {
+    CK(cudaMemcpyAsync(f32_stage, V, (size_t)N * d * 4, cudaMemcpyHostToDevice, h->stream));
+    src = f32_stage;
+  }
+  out->raw = src;
+  out->ld_raw = d;
+  if (bf_buf) {
+    CK(launch_to_bf16(src, N, d, d, bf_buf, pad8(d), h->stream));
+    out->bf = bf_buf;
+    out->ld_bf = pad8(d);
+  }
+  return FFH_OK;
+}
+
+ffh_status gram(ffh_t h, const Staged& V, int64_t N, int64_t d, const float* w_padded, float scale,
+                float* C, float* partial, const GramTables& gt, DevStatus* st) {
+  cudaEvent_t t0 = prof_begin(h);
+  if (h->opt.kernel == 1) {
+    CK(launch_gram_simt(V.raw, h->opt.dtype, N, d, V.ld_raw, w_padded, scale, C, d, h->stream));
+    prof_end(h, PROF_GRAM, t0);
+  } else {
+    cudaEvent_t t1 = t0 ? next_event(h) : nullptr;
+    CK(launch_gram_tc(V.bf, N, d, V.ld_bf, w_padded, scale, C, d, partial, gt.tiles, gt.lut,
+                      gt.plan, st, h->opt.fault, h->stream, t1));
+    prof_end(h, PROF_GRAM, t0, t1);
+  }
+  return FFH_OK;
+}
+
+ffh_status qform(ffh_t h, const Staged& V, int64_t N, int64_t d, const float* Linv,
+                 __nv_bfloat16* Mb, float* q, DevStatus* st) {
+  if (h->opt.kernel == 1) {
+    cudaEvent_t t0 = prof_begin(h);
+    CK(launch_qform_simt(V.raw, h->opt.dtype, N, d, V.ld_raw, Linv, d, q, h->stream));
+    prof_end(h, PROF_QFORM, t0);
+  } else {
+    const int64_t ldm = pad8(d);
+    CK(launch_lower_to_bf16(Linv, d, d, Mb, ldm, h->stream));
+    cudaEvent_t t0 = prof_begin(h);
+    CK(launch_qform_tc(V.bf, N, d, V.ld_bf, Mb, ldm, q, st, h->stream));
+    prof_end(h, PROF_QFORM, t0);
+  }
+  return FFH_OK;
+}
+
+// Cholesky factor and inverse of F (d x d), timed as one region.
+ffh_status chol(ffh_t h, const float* F, int64_t d, float* L, float* Linv, float* work, float* DI,
+                DevStatus* st, int fault) {
+  cudaEvent_t t0 = prof_begin(h);
+  CK(launch_cholesky(F, d, d, L, Linv, work, DI, st, fault, h->stream));
+  prof_end(h, PROF_CHOL, t0);
+  return FFH_OK;
+}
+
+ffh_status setup_tables(ffh_t h, int64_t N, int64_t d, GramTables* gt, int2* tiles_dev,
+                        int* lut_dev) {
+  gt->plan = gram_plan(N, d, num_sms());
+  gt->tiles = tiles_dev;
+  gt->lut = lut_dev;
+  const int64_t nbm = (d + 127) / 128, nbn = (d + 255) / 256;
+  std::vector<int2> tiles((size_t)(nbm * nbn));
+  std::vector<int> lut((size_t)(nbm * nbn));
+  int T = 0;
+  gram_build_tiles(d, tiles.data(), lut.data(), &T);
+  CK(cudaMemcpyAsync(tiles_dev, tiles.data(), sizeof(int2) * T, cudaMemcpyHostToDevice, h->stream));
+  CK(cudaMemcpyAsync(lut_dev, lut.data(), sizeof(int) * lut.size(), cudaMemcpyHostToDevice,
+                     h->stream));
+  CK(cudaStreamSynchronize(h->stream));  // host vectors go out of scope
+  return FFH_OK;
+}
+
+}  // namespace
+
+extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, int64_t n,
+                              int64_t m, int32_t iters, float tol, float* A_out, float* B_out) {
+  if (!h) return FFH_ERR_INVALID_ARG;
+  h->err.clear();
+  ffh_status vs = validate_opt(h);
+  if (vs) return vs;
+  if (!X || !G || !A_out || !B_out) return fail(h, FFH_ERR_INVALID_ARG, "null pointer argument");
+  if (N < 1 || n < 1 || m < 1 || iters < 1)
+    return fail(h, FFH_ERR_INVALID_ARG, "need N, n, m, iters >= 1");
+  if (N > (int64_t)1 << 30) return fail(h, FFH_ERR_INVALID_ARG, "N too large");
+  if (!(tol >= 0.f) || !std::isfinite(tol)) return fail(h, FFH_ERR_INVALID_ARG, "tol must be finite and >= 0");
+  if (h->opt.dtype == FFH_BF16 && (n % 8 || m % 8))
+    return fail(h, FFH_ERR_INVALID_ARG, "bf16 rows must be 16-byte aligned: n, m multiples of 8");
+  if (h->opt.variant == FFH_FROBENIUS)
+    return fail(h, FFH_ERR_UNSUPPORTED, "the Frobenius variant is not in this build");
+  if (N < std::max(n, m) && h->opt.damping == 0.f)
+    return fail(h, FFH_ERR_RANK, "N = %lld < max(n, m) = %lld without damping",
+                (long long)N, (long long)std::max(n, m));
+  const bool tc = h->opt.kernel == 0;
+  const int dtype = h->opt.dtype;
+  const bool x_dev = is_device_ptr(X), g_dev = is_device_ptr(G);
+  const bool init = h->opt.init_A != nullptr;
+  const int64_t D = std::max(n, m);
+  const int64_t Npad = (N + 63) / 64 * 64 + 64;
+  const int nt = (int)((D + 63) / 64);
+
+  GramPlan pn = gram_plan(N, n, num_sms()), pm = gram_plan(N, m, num_sms());
+  auto layout = [&](Carve& c, DevStatus** st, IterRecord** recs, __nv_bfloat16** Xb,
+                    __nv_bfloat16** Gb, float** stage, float** q, float** r, float** A2,
+                    float** B2, float** L, float** Linv, __nv_bfloat16** Mb, float** work,
+                    float** DI, int2** tn, int** ln, int2** tm, int** lm, float** partial,
+                    double** trb) {
+    *st = c.take<DevStatus>(1);
+    *recs = c.take<IterRecord>(iters + 2);
+    const bool xcopy = (dtype == FFH_F32 && tc) || (dtype == FFH_BF16 && !x_dev);
+    const bool gcopy = (dtype == FFH_F32 && tc) || (dtype == FFH_BF16 && !g_dev);
+    *Xb = xcopy ? c.take<__nv_bfloat16>((size_t)N * pad8(n)) : nullptr;
+    *Gb = gcopy ? c.take<__nv_bfloat16>((size_t)N * pad8(m)) : nullptr;
+    const bool host_f32 = dtype == FFH_F32 && (!x_dev || !g_dev);
+    *stage = host_f32 ? c.take<float>((size_t)N * (size_t)((!x_dev && !g_dev) ? (n + m) : D)) : nullptr;
+    *q = c.take<float>(Npad);
+    *r = c.take<float>(Npad);
+    *A2 = c.take<float>((size_t)2 * n * n);
+    *B2 = c.take<float>((size_t)2 * m * m);
+    *L = c.take<float>((size_t)D * D);
+    *Linv = c.take<float>((size_t)D * D);
+    *Mb = c.take<__nv_bfloat16>((size_t)D * pad8(D));
+    *work = c.take<float>(cholesky_work_floats(D));
+    *DI = c.take<float>((size_t)nt * 64 * 64);
+    *tn = c.take<int2>(gram_tile_table_bytes(n) / sizeof(int2) + 1);
+    *ln = c.take<int>(gram_tile_table_bytes(n) / sizeof(int) + 1);
+    *tm = c.take<int2>(gram_tile_table_bytes(m) / sizeof(int2) + 1);
+    *lm = c.take<int>(gram_tile_table_bytes(m) / sizeof(int) + 1);
+    *partial = tc ? c.take<float>(std::max(gram_partial_bytes(pn), gram_partial_bytes(pm)) / 4)
+                  : nullptr;
+    *trb = c.take<double>(8);
+  };
+  DevStatus* st;
+  IterRecord* recs;
+  __nv_bfloat16 *Xb, *Gb, *Mb;
+  float *stage, *q, *r, *A2, *B2, *L, *Linv, *work, *DI, *partial;
+  int2 *tn, *tm;
+  int *ln, *lm;
+  double* trb;
+  {
+    Carve c(nullptr);
+    layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &DI, &tn,
+           &ln, &tm, &lm, &partial, &trb);
+    ffh_status es = ensure_ws(h, c.off + 1024);
+    if (es) return es;
+  }
+  Carve c(h->ws);
+  layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &DI, &tn, &ln,
+         &tm, &lm, &partial, &trb);
+  cudaStream_t s = h->stream;
+  CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
+  CK(cudaMemsetAsync(recs, 0, sizeof(IterRecord) * (iters + 2), s));
+  CK(cudaMemsetAsync(q, 0, sizeof(float) * Npad, s));
+  CK(cudaMemsetAsync(r, 0, sizeof(float) * Npad, s));
+  GramTables gtn, gtm;
+  if (tc) {
+    ffh_status es = setup_tables(h, N, n, &gtn, tn, ln);
+    if (es) return es;
+    es = setup_tables(h, N, m, &gtm, tm, lm);
+    if (es) return es;
+  }
+  Staged xs, gs;
+  ffh_status es = stage_input(h, X, x_dev, N, n, Xb, stage, &xs);
+  if (es) return es;
+  // both host fp32: X and G get separate staging regions
+  float* stage_g = stage ? ((!x_dev && !g_dev) ? stage + (size_t)N * n : stage) : nullptr;
+  es = stage_input(h, G, g_dev, N, m, Gb, stage_g, &gs);
+  if (es) return es;
+
+  float* A[2] = {A2, A2 + (size_t)n * n};
+  float* B[2] = {B2, B2 + (size_t)m * m};
+  int cur = 0;
+  if (init) {
+    CK(cudaMemcpyAsync(A[cur], h->opt.init_A, sizeof(float) * n * n, cudaMemcpyDefault, s));
+  } else {
+    CK(launch_fill_identity(A[cur], n, n, s));
+  }
+  const float lam = h->opt.damping;
+  const float sB = (float)(1.0 / ((double)N * (double)n));
+  const float sA = (float)(1.0 / ((double)N * (double)m));
+  int t_done = 0;
+  std::vector<IterRecord> host_recs((size_t)iters + 2);
+  for (int t = 1; t <= iters; ++t) {
+    IterRecord* R = recs + t;
+    const int nxt = cur ^ 1;
+    // ---- weights q_k = x_k^T A_{t-1}^-1 x_k
+    if (t == 1 && !init) {
+      CK(launch_rowsumsq(xs.raw, dtype, N, n, xs.ld_raw, q, s));
+    } else {
+      es = chol(h, A[cur], n, L, Linv, work, DI, st, 0);
+      if (es) return es;
+      CK(cudaMemcpyAsync(&R->logdet_A_prev, &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
+      if (t > 1)
+        CK(cudaMemcpyAsync(&recs[t - 1].logdet_A, &st->logdet, sizeof(double),
+                           cudaMemcpyDeviceToDevice, s));
+      es = qform(h, xs, N, n, Linv, Mb, q, st);
+      if (es) return es;
+      if (t > 1) CK(launch_dot(q, r, N, &recs[t - 1].sum_qr_A, s));
+    }
+    // ---- B-update
+    es = gram(h, gs, N, m, q, sB, B[nxt], partial, gtm, st);
+    if (es) return es;
+    CK(launch_damp(B[nxt], m, m, lam, st, s));
+    es = chol(h, B[nxt], m, L, Linv, work, DI, st,
+              (t == 1 && h->opt.fault == FFH_FAULT_BAD_PIVOT) ? FFH_FAULT_BAD_PIVOT : 0);
+    if (es) return es;
+    CK(cudaMemcpyAsync(&R->logdet_B, &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
+    es = qform(h, gs, N, m, Linv, Mb, r, st);
+    if (es) return es;
+    CK(launch_dot(q, r, N, &R->sum_qr_B, s));
+    // ---- A-update
+    es = gram(h, xs, N, n, r, sA, A[nxt], partial, gtn, st);
+    if (es) return es;
+    CK(launch_damp(A[nxt], n, n, lam, st, s));
+    CK(launch_normalize(A[nxt], n, B[nxt], m, R, st, s));
+    // ---- convergence statistics
+    CK(cudaMemsetAsync(&R->dA2, 0, sizeof(double) * 4, s));
+    CK(launch_trace(A[nxt], n, trb + 0, s));
+    CK(launch_trace(A[cur], n, trb + 1, s));
+    CK(launch_delta(A[nxt], A[cur], n, &R->dA2, &R->nA2, trb, s));
+    if (t > 1) {
+      CK(launch_trace(B[nxt], m, trb + 2, s));
+      CK(launch_trace(B[cur], m, trb + 3, s));
+      CK(launch_delta(B[nxt], B[cur], m, &R->dB2, &R->nB2, trb + 2, s));
+    }
+    cur = nxt;
+    t_done = t;
+    if (tol > 0.f && t > 1) {
+      IterRecord hr;
+      CK(cudaMemcpyAsync(&hr, R, sizeof(hr), cudaMemcpyDeviceToHost, s));
+      CK(cudaStreamSynchronize(s));
+      const double dA = hr.nA2 > 0 ? std::sqrt(hr.dA2 / hr.nA2) : 0.0;
+      const double dB = hr.nB2 > 0 ? std::sqrt(hr.dB2 / hr.nB2) : 0.0;
+      if (std::max(dA, dB) < (double)tol) break;
+    }
+  }
+  if (h->opt.final_loglik) {
+    es = chol(h, A[cur], n, L, Linv, work, DI, st, 0);
+    if (es) return es;
+    CK(cudaMemcpyAsync(&recs[t_done].logdet_A, &st->logdet, sizeof(double),
+                       cudaMemcpyDeviceToDevice, s));
+    es = qform(h, xs, N, n, Linv, Mb, q, st);
+    if (es) return es;
+    CK(launch_dot(q, r, N, &recs[t_done].sum_qr_A, s));
+  }
+  CK(cudaMemcpyAsync(A_out, A[cur], sizeof(float) * n * n, cudaMemcpyDefault, s));
+  CK(cudaMemcpyAsync(B_out, B[cur], sizeof(float) * m * m, cudaMemcpyDefault, s));
+  CK(cudaMemcpyAsync(host_recs.data(), recs, sizeof(IterRecord) * (iters + 2),
+                     cudaMemcpyDeviceToHost, s));
+  es = read_status(h, st);
+  h->iters_done = t_done;
+  h->N = N;
+  h->n = n;
+  h->m = m;
+  h->final_loglik = h->opt.final_loglik != 0;
+  h->recs = host_recs;
+  return es;
+}
+
+extern "C" ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_t n, int64_t m,
+                                     int32_t iters, float tol, float* A_out, float* B_out) {
+  if (!h) return FFH_ERR_INVALID_ARG;
+  (void)Gk;
+  (void)N;
+  (void)n;
+  (void)m;
+  (void)iters;
+  (void)tol;
+  (void)A_out;
+  (void)B_out;
+  return fail(h, FFH_ERR_UNSUPPORTED, "matrix-sample fit is not in this build");
+}
+
+extern "C" ffh_status ffh_get_stats(ffh_t h, int32_t* iters_done, double* delta,
+                                    double* loglik_trace, double* mean_qr, int32_t capacity,
+                                    int32_t* n_trace) {
+  if (!h) return FFH_ERR_INVALID_ARG;
+  const int T = h->iters_done;
+  if (iters_done) *iters_done = T;
+  if (n_trace) *n_trace = 2 * T;
+  const double N = (double)h->N, n = (double)h->n, m = (double)h->m;
+  if (delta) {
+    if (T <= 1 || h->recs.empty()) {
+      *delta = INFINITY;
+    } else {
+      const IterRecord& R = h->recs[T];
+      const double dA = R.nA2 > 0 ? std::sqrt(R.dA2 / R.nA2) : 0.0;
+      const double dB = R.nB2 > 0 ? std::sqrt(R.dB2 / R.nB2) : 0.0;
+      *delta = std::max(dA, dB);
+    }
+  }
+  for (int t = 1; t <= T; ++t) {
+    const IterRecord& R = h->recs[t];
+    const int i0 = 2 * (t - 1), i1 = i0 + 1;
+    // l(A_{t-1}, B_t): B_t before the rescale, r computed with it
+    const double lB = -0.5 * (N * m * R.logdet_A_prev + N * n * R.logdet_B + R.sum_qr_B);
+    // l(A_t, B_t) after the rescale s: log|sB| = log|B| + m log s, r/s
+    const bool haveA = t < T || h->final_loglik;
+    const double ldB_s = R.logdet_B + m * std::log(R.scale);
+    const double lA = haveA ? -0.5 * (N * m * R.logdet_A + N * n * ldB_s + R.sum_qr_A / R.scale)
+                            : NAN;
+    if (loglik_trace) {
+      if (i0 < capacity) loglik_trace[i0] = lB;
+      if (i1 < capacity) loglik_trace[i1] = lA;
+    }
+    if (mean_qr) {
+      if (i0 < capacity) mean_qr[i0] = R.sum_qr_B / N;
+      if (i1 < capacity) mean_qr[i1] = haveA ? R.sum_qr_A / (N * R.scale) : NAN;
+    }
+  }
+  return FFH_OK;
+}
+
+// ---------------------------------------------------------------------------
+// single steps
+// ---------------------------------------------------------------------------
+extern "C" ffh_status ffh_weighted_gram(ffh_t h, const void* V, const float* w, int64_t N,
+                                        int64_t d, float scale, float* C_out) {
+  if (!h) return FFH_ERR_INVALID_ARG;
+  h->err.clear();
+  ffh_status vs = validate_opt(h);
+  if (vs) return vs;
+  if (!V || !C_out || N < 1 || d < 1) return fail(h, FFH_ERR_INVALID_ARG, "bad arguments");
+  if (N > (int64_t)1 << 30) return fail(h, FFH_ERR_INVALID_ARG, "N too large");
+  if (!is_device_ptr(V) || !is_device_ptr(C_out) || (w && !is_device_ptr(w)))
+    return fail(h, FFH_ERR_INVALID_ARG, "single-step calls take device pointers");
+  const int dtype = h->opt.dtype;
+  if (dtype == FFH_BF16 && d % 8) return fail(h, FFH_ERR_INVALID_ARG, "bf16 rows: d multiple of 8");
+  const bool tc = h->opt.kernel == 0;
+  const int64_t Npad = (N + 63) / 64 * 64 + 64;
+  GramPlan plan = gram_plan(N, d, num_sms());
+  auto layout = [&](Carve& c, DevStatus** st, float** wp, __nv_bfloat16** Vb, float** partial,
+                    int2** tiles, int** lut) {
+    *st = c.take<DevStatus>(1);
+    *wp = c.take<float>(Npad);
+    *Vb = (tc && dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(d)) : nullptr;
+    *partial = tc ? c.take<float>(gram_partial_bytes(plan) / 4) : nullptr;
+    *tiles = c.take<int2>(gram_tile_table_bytes(d) / sizeof(int2) + 1);
+    *lut = c.take<int>(gram_tile_table_bytes(d) / sizeof(int) + 1);
+  };
+  DevStatus* st;
+  float *wp, *partial;
+  __nv_bfloat16* Vb;
+  int2* tiles;
+  int* lut;
+  {
+    Carve c(nullptr);
+    layout(c, &st, &wp, &Vb, &partial, &tiles, &lut);
+    ffh_status es = ensure_ws(h, c.off + 1024);
+    if (es) return es;
+  }
+  Carve c(h->ws);
+  layout(c, &st, &wp, &Vb, &partial, &tiles, &lut);
+  cudaStream_t s = h->stream;
+  CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
+  const float* wuse = nullptr;
+  if (w) {
+    CK(cudaMemsetAsync(wp, 0, sizeof(float) * Npad, s));
+    CK(cudaMemcpyAsync(wp, w, sizeof(float) * N, cudaMemcpyDeviceToDevice, s));
+    wuse = wp;
+  }
+  Staged vs_;
+  ffh_status es = stage_input(h, V, true, N, d, Vb, nullptr, &vs_);
+  if (es) return es;
+  GramTables gt;
+  if (tc) {
+    es = setup_tables(h, N, d, &gt, tiles, lut);
+    if (es) return es;
+  }
+  es = gram(h, vs_, N, d, wuse, scale, C_out, partial, gt, st);
+  if (es) return es;
+  return read_status(h, st);
+}
+
+extern "C" ffh_status ffh_quad_form(ffh_t h, const void* V, const float* Linv, int64_t N,
+                                    int64_t d, float* q_out) {
+  if (!h) return FFH_ERR_INVALID_ARG;
+  h->err.clear();
+  ffh_status vs = validate_opt(h);
+  if (vs) return vs;
+  if (!V || !Linv || !q_out || N < 1 || d < 1) return fail(h, FFH_ERR_INVALID_ARG, "bad arguments");
+  if (N > (int64_t)1 << 30) return fail(h, FFH_ERR_INVALID_ARG, "N too large");
+  if (!is_device_ptr(V) || !is_device_ptr(Linv) || !is_device_ptr(q_out))
+    return fail(h, FFH_ERR_INVALID_ARG, "single-step calls take device pointers");
+  const int dtype = h->opt.dtype;
+  if (dtype == FFH_BF16 && d % 8) return fail(h, FFH_ERR_INVALID_ARG, "bf16 rows: d multiple of 8");
+  const bool tc = h->opt.kernel == 0;
+  auto layout = [&](Carve& c, DevStatus** st, __nv_bfloat16** Vb, __nv_bfloat16** Mb) {
+    *st = c.take<DevStatus>(1);
+    *Vb = (tc && dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(d)) : nullptr;
+    *Mb = c.take<__nv_bfloat16>((size_t)d * pad8(d));
+  };
+  DevStatus* st;
+  __nv_bfloat16 *Vb, *Mb;
+  {
+    Carve c(nullptr);
+    layout(c, &st, &Vb, &Mb);
+    ffh_status es = ensure_ws(h, c.off + 1024);
+    if (es) return es;
+  }
+  Carve c(h->ws);
+  layout(c, &st, &Vb, &Mb);
+  CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), h->stream));
+  Staged vs_;
+  ffh_status es = stage_input(h, V, true, N, d, Vb, nullptr, &vs_);
+  if (es) return es;
+  es = qform(h, vs_, N, d, Linv, Mb, q_out, st);
+  if (es) return es;
+  return read_status(h, st);
+}
+
+extern "C" ffh_status ffh_cholesky(ffh_t h, const float* F, int64_t d, float* L_out,
+                                   float* Linv_out, double* logdet) {
+  if (!h) return FFH_ERR_INVALID_ARG;
+  h->err.clear();
+  if (!F || d < 1) return fail(h, FFH_ERR_INVALID_ARG, "bad arguments");
+  if (!is_device_ptr(F) || (L_out && !is_device_ptr(L_out)) ||
+      (Linv_out && !is_device_ptr(Linv_out)))
+    return fail(h, FFH_ERR_INVALID_ARG, "single-step calls take device pointers");
+  const int nt = (int)((d + 63) / 64);
+  auto layout = [&](Carve& c, DevStatus** st, float** L, float** Li, float** work, float** DI) {
+    *st = c.take<DevStatus>(1);
+    *L = L_out ? nullptr : c.take<float>((size_t)d * d);
+    *Li = c.take<float>((size_t)d * d);
+    *work = c.take<float>(cholesky_work_floats(d));
+    *DI = c.take<float>((size_t)nt * 64 * 64);
+  };
+  DevStatus* st;
+  float *L, *Li, *work, *DI;
+  {
+    Carve c(nullptr);
+    layout(c, &st, &L, &Li, &work, &DI);
+    ffh_status es = ensure_ws(h, c.off + 1024);
+    if (es) return es;
+  }
+  Carve c(h->ws);
+  layout(c, &st, &L, &Li, &work, &DI);
+  if (L_out) L = L_out;
+  cudaStream_t s = h->stream;
+  CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
+  ffh_status cs = chol(h, F, d, L, Linv_out ? Linv_out : (float*)nullptr, work, DI, st,
+                       h->opt.fault == FFH_FAULT_BAD_PIVOT ? FFH_FAULT_BAD_PIVOT : 0);
+  if (cs) return cs;
+  (void)Li;
+  DevStatus hst;
+  CK(cudaMemcpyAsync(&hst, st, sizeof(hst), cudaMemcpyDeviceToHost, s));
+  ffh_status es = read_status(h, st);
+  if (logdet) *logdet = hst.logdet;
+  return es;
+}
+
+extern "C" ffh_status ffh_get_timings(ffh_t h, ffh_timings* out, int32_t reset) {
+  if (!h || !out) return FFH_ERR_INVALID_ARG;
+  if (!h->pending.empty()) {
+    CK(cudaStreamSynchronize(h->stream));
+    prof_resolve(h);
+  }
+  out->gram_ms = h->prof_ms[PROF_GRAM];
+  out->gram_launches = h->prof_n[PROF_GRAM];
+  out->qform_ms = h->prof_ms[PROF_QFORM];
+  out->qform_launches = h->prof_n[PROF_QFORM];
+  out->chol_ms = h->prof_ms[PROF_CHOL];
+  out->chol_calls = h->prof_n[PROF_CHOL];
+  out->kernel_launches = launches_so_far();
+  if (reset) {
+    for (int k = 0; k < 3; ++k) {
+      h->prof_ms[k] = 0;
+      h->prof_n[k] = 0;
+    }
+  }
+  return FFH_OK;
+}

@@ -1,0 +1,109 @@
+// Internal declarations shared by the libffh translation units.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/ffh.h"
+
+namespace ffh {
+
+// ---------------------------------------------------------------------------
+// device status block (one per handle, in the workspace)
+// ---------------------------------------------------------------------------
+struct DevStatus {
+  int error;        // first FFH_ERR_* raised by a kernel (0 = none)
+  int error_info;   // where: pivot index, or timeout site
+  int abort_all;    // set together with error; kernels test it on entry
+  int pad;
+  double logdet;    // log|F| of the last Cholesky
+  double acc[8];    // scratch reductions (traces, norms, dot products)
+};
+
+// per-iteration record kept on the device, read once at the end of a fit
+struct IterRecord {
+  double logdet_A_prev;  // log|A_{t-1}| (after normalisation)
+  double logdet_B;       // log|B_t| before the A-side rescale
+  double sum_qr_B;       // sum_k q_k r_k at (A_{t-1}, B_t)
+  double sum_qr_A;       // sum_k q_k r_k at (A_t, B_t) (filled by the next iteration)
+  double logdet_A;       // log|A_t| (filled by the next iteration)
+  double scale;          // s = tr(A_t)/n before normalisation
+  double dA2, nA2;       // ||A^_t - A^_{t-1}||^2, ||A^_t||^2
+  double dB2, nB2;       // same for B
+  double trB;            // tr(B_t) after the rescale
+  double pad;
+};
+
+__device__ __forceinline__ void raise_error(DevStatus* st, int code, int info) {
+  if (atomicCAS(&st->error, 0, code) == 0) {
+    st->error_info = info;
+  }
+  atomicExch(&st->abort_all, 1);
+}
+
+// ---------------------------------------------------------------------------
+// launch helpers (host)
+// ---------------------------------------------------------------------------
+struct Ctx;  // defined in ffh_api.cu
+
+int num_sms();
+// process-wide count of kernels launched by libffh
+void note_launches(int k);
+long long launches_so_far();
+
+// tensor-core kernels (kernels_tc.cu)
+struct GramPlan {
+  int T;        // lower-triangle output tiles
+  int S;        // K splits
+  int KB;       // 64-sample blocks
+  int units;    // T * S
+  int grid;     // persistent CTAs
+};
+GramPlan gram_plan(int64_t N, int64_t d, int sms);
+size_t gram_partial_bytes(const GramPlan& p);
+// C = scale * V^T diag(w) V (lower tiles, then mirrored), V bf16 N x d (pitch ld elements)
+cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t ld,
+                           const float* w_padded, float scale, float* C, int64_t ldc,
+                           float* partial, int2* tiles_dev, int* tile_lut_dev,
+                           const GramPlan& plan, DevStatus* st, int fault, cudaStream_t s,
+                           cudaEvent_t after_main = nullptr);
+// q_k = ||M v_k||^2, V bf16 N x d (pitch ld), M bf16 d x d lower (pitch ldm)
+cudaError_t launch_qform_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t ld,
+                            const __nv_bfloat16* M, int64_t ldm, float* q, DevStatus* st,
+                            cudaStream_t s);
+size_t gram_tile_table_bytes(int64_t d);
+void gram_build_tiles(int64_t d, int2* tiles_host, int* lut_host, int* T_out);
+
+// CUDA-core kernels (kernels_simt.cu)
+cudaError_t launch_gram_simt(const void* V, int dtype, int64_t N, int64_t d, int64_t ld,
+                             const float* w, float scale, float* C, int64_t ldc, cudaStream_t s);
+cudaError_t launch_qform_simt(const void* V, int dtype, int64_t N, int64_t d, int64_t ld,
+                              const float* M, int64_t ldm, float* q, cudaStream_t s);
+cudaError_t launch_fwd_qform_simt(const void* V, int dtype, int64_t N, int64_t d, int64_t ld,
+                                  const float* F, int64_t ldf, float* q, cudaStream_t s);
+cudaError_t launch_rowsumsq(const void* V, int dtype, int64_t N, int64_t d, int64_t ld, float* q,
+                            cudaStream_t s);
+cudaError_t launch_to_bf16(const float* src, int64_t rows, int64_t cols, int64_t lds,
+                           __nv_bfloat16* dst, int64_t ldd, cudaStream_t s);
+// Cholesky L (lower, fp32), L^-1 (fp32, lower), logdet accumulated into st->logdet
+cudaError_t launch_cholesky(const float* F, int64_t d, int64_t ldf, float* L, float* Linv,
+                            float* work, float* diag_inv, DevStatus* st, int fault,
+                            cudaStream_t s);
+size_t cholesky_work_floats(int64_t d);
+cudaError_t launch_fill_identity(float* F, int64_t d, int64_t ld, cudaStream_t s);
+cudaError_t launch_damp(float* F, int64_t d, int64_t ld, float lambda, DevStatus* st,
+                        cudaStream_t s);
+// A <- A / s, B <- B * s with s = tr(A)/n; records s and log-determinant corrections
+cudaError_t launch_normalize(float* A, int64_t n, float* B, int64_t m, IterRecord* rec,
+                             DevStatus* st, cudaStream_t s);
+cudaError_t launch_delta(const float* F, const float* Fprev, int64_t d, double* d2, double* n2,
+                         double* tr, cudaStream_t s);
+cudaError_t launch_dot(const float* a, const float* b, int64_t N, double* out, cudaStream_t s);
+cudaError_t launch_frob2(const float* F, int64_t d, double* out, cudaStream_t s);
+cudaError_t launch_scale_by_inv(float* F, int64_t d, const double* denom, cudaStream_t s);
+cudaError_t launch_copy_logdet(DevStatus* st, double* dst, cudaStream_t s);
+cudaError_t launch_zero_f64(double* p, int n, cudaStream_t s);
+
+}  // namespace ffh

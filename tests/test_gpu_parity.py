@@ -1,0 +1,252 @@
+"""Parity of the CUDA path (through the C ABI) with the fp64 oracle.
+
+Tolerances are derived from the arithmetic of each step:
+  * weighted Gram: the weighted operand is rounded to bf16 once (relative error
+    <= 2^-9 per term) and accumulated in fp32, so elementwise
+    |C - C_ref| <= 2^-8 * (|V|^T diag(|w|) |V|) * scale   (2^-8 leaves room for the
+    fp32 accumulation, whose error is orders of magnitude smaller for N <= 2^19);
+  * quadratic form: L^-1 is rounded to bf16 (2^-9 per entry), inputs are exact,
+    so with y = L^-1 v, z = |L^-1| |v|:  |q - q_ref| <= 2^-8 sum_i |y_i| z_i
+    + 2^-18 sum_i z_i^2 (plus fp32 accumulation);
+  * the fit: relative Frobenius error of the trace-normalised A (x) B <= 2e-3.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2609_14706_gb300 as ffh
+import synth
+
+pytestmark = pytest.mark.gpu
+
+KERNELS = ["tc", "simt"]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    from paper_2609_14706_gb300 import build
+    build.build()
+
+
+def _bf16_gram_bound(V, w, scale):
+    Va = np.abs(V)
+    wa = np.ones(V.shape[0]) if w is None else np.abs(w)
+    return 2.0 ** -8 * scale * ((Va.T * wa) @ Va)
+
+
+# ---------------------------------------------------------------------------
+# weighted Gram
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("kernel", KERNELS)
+@pytest.mark.parametrize("N,d,weighted", [(1000, 64, True), (5000, 320, True), (4097, 136, False),
+                                          (3000, 512, True), (700, 8, True)])
+def test_weighted_gram_matches_oracle(kernel, N, d, weighted):
+    wl = synth.WORKLOADS["llama7b_attn_4096"].with_(n=d, m=8)
+    X, _ = synth.rank_one_samples(wl, seed=1, device="cuda", N=N)
+    w = (torch.rand(N, device="cuda", generator=torch.Generator("cuda").manual_seed(2)) * 3
+         if weighted else None)
+    scale = 1.0 / (N * 7)
+    with ffh.Handle(dtype="bf16", kernel=kernel) as h:
+        C = h.weighted_gram(X, w, scale)
+    torch.cuda.synchronize()
+    Vn = oracle.as_f64(X)
+    wn = None if w is None else oracle.as_f64(w)
+    ref = oracle.weighted_gram(Vn, np.ones(N) if wn is None else wn, scale)
+    Cn = oracle.as_f64(C)
+    assert np.array_equal(Cn, Cn.T), "output must be exactly symmetric"
+    bound = _bf16_gram_bound(Vn, wn, scale) + 1e-7 * np.abs(ref).max()
+    assert np.all(np.abs(Cn - ref) <= bound), np.max(np.abs(Cn - ref) / bound)
+
+
+def test_weighted_gram_f32_input():
+    N, d = 2000, 100          # fp32 input: any d (internally padded to a multiple of 8)
+    X = synth.gaussian(N, d, seed=3, device="cuda")
+    w = torch.rand(N, device="cuda")
+    with ffh.Handle(dtype="f32") as h:
+        C = h.weighted_gram(X, w, 0.5)
+    Vn, wn = oracle.as_f64(X), oracle.as_f64(w)
+    ref = oracle.weighted_gram(Vn, wn, 0.5)
+    # fp32 inputs are rounded to bf16 on both operands: 2 * 2^-9 + 2^-9
+    bound = 3 * 2.0 ** -9 * 0.5 * ((np.abs(Vn).T * wn) @ np.abs(Vn)) + 1e-7 * np.abs(ref).max()
+    assert np.all(np.abs(oracle.as_f64(C) - ref) <= bound)
+
+
+# ---------------------------------------------------------------------------
+# quadratic form
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("kernel", KERNELS)
+@pytest.mark.parametrize("N,d", [(1000, 64), (3000, 264), (1500, 512), (129, 1024)])
+def test_quad_form_matches_oracle(kernel, N, d):
+    wl = synth.WORKLOADS["llama7b_attn_4096"].with_(n=d, m=8)
+    X, _ = synth.rank_one_samples(wl, seed=4, device="cuda", N=N)
+    A = oracle.as_f64(synth.spd_matrix(d, seed=5, cond=1e3, dtype=torch.float64))
+    Linv = oracle.tri_inverse(oracle.cholesky(A))
+    with ffh.Handle(dtype="bf16", kernel=kernel) as h:
+        q = h.quad_form(X, torch.tensor(Linv, dtype=torch.float32, device="cuda"))
+    Xn = oracle.as_f64(X)
+    ref = oracle.inv_quad_forms_chol(oracle.cholesky(A), Xn)
+    Lf = Linv.astype(np.float32).astype(np.float64)   # what the kernel is given
+    y = Xn @ Lf.T
+    z = np.abs(Xn) @ np.abs(Lf).T
+    bound = (2.0 ** -8 * np.sum(np.abs(y) * z, 1) + 2.0 ** -18 * np.sum(z * z, 1)
+             + 1e-5 * ref + np.abs(np.sum(y * y, 1) - ref))
+    assert np.all(np.abs(oracle.as_f64(q) - ref) <= bound)
+
+
+# ---------------------------------------------------------------------------
+# Cholesky and inverse
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("d,cond", [(64, 1e2), (200, 1e3), (512, 1e3), (1000, 1e4), (1536, 1e3)])
+def test_cholesky_matches_oracle(d, cond):
+    A = synth.spd_matrix(d, seed=6, cond=cond, dtype=torch.float32, device="cuda")
+    with ffh.Handle() as h:
+        L, Li, logdet = h.cholesky(A)
+    An = oracle.as_f64(A)
+    Lr = oracle.cholesky(An)
+    Mr = oracle.tri_inverse(Lr)
+    eps = 2.0 ** -24
+    assert np.allclose(np.triu(oracle.as_f64(L), 1), 0)
+    assert np.allclose(np.triu(oracle.as_f64(Li), 1), 0)
+    eL = np.linalg.norm(oracle.as_f64(L) - Lr) / np.linalg.norm(Lr)
+    eM = np.linalg.norm(oracle.as_f64(Li) - Mr) / np.linalg.norm(Mr)
+    # backward-stable fp32 Cholesky: forward error ~ d * eps * cond
+    assert eL <= 4 * d * eps * cond, eL
+    assert eM <= 8 * d * eps * cond, eM
+    assert logdet == pytest.approx(oracle.logdet_from_cholesky(Lr), rel=1e-5, abs=1e-3)
+
+
+def test_cholesky_rejects_indefinite():
+    A = torch.eye(100, device="cuda")
+    A[50, 50] = -1.0
+    with ffh.Handle() as h:
+        with pytest.raises(ffh.FFHError) as ei:
+            h.cholesky(A)
+    assert ei.value.status == "FFH_ERR_NOT_SPD" and "50" in str(ei.value)
+
+
+# ---------------------------------------------------------------------------
+# the fit
+# ---------------------------------------------------------------------------
+FIT_CASES = {
+    # the tiny rank-one configuration exactly (fp32, 10 iterations)
+    "tiny_64": synth.WORKLOADS["tiny_64"],
+    # bf16 LLM-like samples at a size the oracle finishes in seconds; m ragged vs 256
+    "llama_small": synth.WORKLOADS["llama7b_attn_4096"].with_(N=16384, n=256, m=320, iters=4),
+    # heavy-tailed inputs, n > m
+    "student_small": synth.WORKLOADS["llama3_8b_down_14336x4096"].with_(N=20000, n=448, m=128,
+                                                                        iters=4),
+}
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+@pytest.mark.parametrize("case", sorted(FIT_CASES))
+def test_fit_matches_oracle(case, kernel):
+    wl = FIT_CASES[case]
+    X, G = synth.rank_one_samples(wl, seed=0, device="cuda")
+    with ffh.Handle(dtype=wl.dtype, kernel=kernel, final_loglik=True) as h:
+        A, B = h.fit(X, G, iters=wl.iters)
+        st = h.stats()
+    ref = oracle.flipflop_fit(X.cpu(), G.cpu(), iters=wl.iters)
+    err = oracle.kron_rel_err(A.cpu(), B.cpu(), ref.A, ref.B)
+    assert err <= 2e-3, err
+    An = oracle.as_f64(A)
+    assert np.trace(An) == pytest.approx(wl.n, rel=1e-4)
+    assert np.array_equal(An, An.T)
+    assert st["iters_done"] == wl.iters
+    n, m = wl.n, wl.m
+    # trace identity mean_k q_k r_k = m n after every half-step
+    assert np.allclose(st["mean_qr"], m * n, rtol=2e-2)
+    # log-likelihood: matches the oracle's trace and is non-decreasing
+    ll = np.array(st["loglik"])
+    assert np.allclose(ll, ref.loglik, rtol=1e-3, atol=1e-3 * np.abs(ref.loglik).max())
+
+
+def test_fit_factorial_design_closed_form():
+    """GPU fit of a factorial design reaches A (x) B = Sigma_x (x) Sigma_g."""
+    P, R, n, m = 256, 128, 256, 128
+    X, G, Xp, Gr = synth.factorial_design(P, R, n, m, seed=7, device="cuda", dtype=torch.bfloat16)
+    Xp, Gr = oracle.as_f64(Xp), oracle.as_f64(Gr)
+    Sx, Sg = Xp.T @ Xp / P, Gr.T @ Gr / R
+    with ffh.Handle(dtype="bf16") as h:
+        A, B = h.fit(X, G, iters=2)
+    assert oracle.kron_rel_err(A.cpu(), B.cpu(), Sx, Sg) <= 2e-3
+
+
+def test_fit_host_inputs_equal_device_inputs():
+    wl = FIT_CASES["llama_small"].with_(iters=2)
+    X, G = synth.rank_one_samples(wl, seed=0, device="cuda")
+    with ffh.Handle(dtype="bf16") as h:
+        A1, B1 = h.fit(X, G, iters=2)
+        A2, B2 = h.fit(X.cpu().pin_memory(), G.cpu(), iters=2)
+    assert torch.equal(A1.cpu(), A2) and torch.equal(B1.cpu(), B2)
+
+
+def test_fit_damping_matches_oracle():
+    wl = FIT_CASES["llama_small"].with_(iters=3)
+    X, G = synth.rank_one_samples(wl, seed=0, device="cuda")
+    with ffh.Handle(dtype="bf16", damping=0.1) as h:
+        A, B = h.fit(X, G, iters=3)
+    ref = oracle.flipflop_fit(X.cpu(), G.cpu(), iters=3, damping=0.1)
+    assert oracle.kron_rel_err(A.cpu(), B.cpu(), ref.A, ref.B) <= 2e-3
+
+
+def test_fit_tol_stops_early():
+    wl = FIT_CASES["tiny_64"]
+    X, G = synth.rank_one_samples(wl, seed=0, device="cuda")
+    with ffh.Handle(dtype="f32") as h:
+        h.fit(X, G, iters=50, tol=1e-4)
+        st = h.stats()
+    ref = oracle.flipflop_fit(X.cpu(), G.cpu(), iters=50, tol=1e-4)
+    assert st["iters_done"] < 50 and st["delta"] < 1e-4
+    assert abs(st["iters_done"] - ref.iters_done) <= 1
+
+
+def test_fit_warm_start():
+    wl = FIT_CASES["llama_small"].with_(iters=2)
+    X, G = synth.rank_one_samples(wl, seed=0, device="cuda")
+    ref1 = oracle.flipflop_fit(X.cpu(), G.cpu(), iters=1)
+    ref3 = oracle.flipflop_fit(X.cpu(), G.cpu(), iters=2, init_A=ref1.A)
+    A0 = torch.tensor(ref1.A, dtype=torch.float32, device="cuda")
+    with ffh.Handle(dtype="bf16", init_A=A0) as h:
+        A, B = h.fit(X, G, iters=2)
+    assert oracle.kron_rel_err(A.cpu(), B.cpu(), ref3.A, ref3.B) <= 2e-3
+
+
+# ---------------------------------------------------------------------------
+# errors
+# ---------------------------------------------------------------------------
+def test_fit_argument_errors():
+    X = torch.zeros(100, 16, dtype=torch.bfloat16, device="cuda")
+    G = torch.zeros(100, 12, dtype=torch.bfloat16, device="cuda")
+    with ffh.Handle(dtype="bf16") as h:
+        with pytest.raises(ffh.FFHError) as ei:
+            h.fit(X, G, iters=1)          # m = 12 is not a multiple of 8
+        assert ei.value.status == "FFH_ERR_INVALID_ARG"
+        with pytest.raises(ffh.FFHError) as ei:
+            h.fit(X[:10], X[:10], iters=1)
+        assert ei.value.status == "FFH_ERR_RANK"
+        with pytest.raises(ffh.FFHError) as ei:
+            h.fit(X, X, iters=0)
+        assert ei.value.status == "FFH_ERR_INVALID_ARG"
+
+
+def test_fault_injection_oom_and_pivot():
+    wl = FIT_CASES["llama_small"].with_(iters=2)
+    X, G = synth.rank_one_samples(wl, seed=0, device="cuda")
+    with ffh.Handle(dtype="bf16", fault=ffh.FAULT_OOM) as h:
+        with pytest.raises(ffh.FFHError) as ei:
+            h.fit(X, G, iters=2)
+        assert ei.value.status == "FFH_ERR_OOM"
+    with ffh.Handle(dtype="bf16", fault=ffh.FAULT_BAD_PIVOT) as h:
+        with pytest.raises(ffh.FFHError) as ei:
+            h.fit(X, G, iters=2)
+        assert ei.value.status == "FFH_ERR_NOT_SPD"
+    # the context is still usable afterwards
+    with ffh.Handle(dtype="bf16") as h:
+        A, B = h.fit(X, G, iters=1)
+    assert torch.isfinite(A).all()
