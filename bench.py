@@ -1,0 +1,330 @@
+#!/usr/bin/env python
+"""Benchmark of the FlipFlop Hessian fit on GB300.
+
+One step = one full fit of the workload (A_0 = I, `iters` flip-flop iterations,
+tol = 0): every stage of the path (initial weights, Cholesky, inverse, quadratic
+forms, weighted Grams, normalisation, convergence statistics) runs inside the
+timed region, through the libffh C ABI.  The headline workload is the
+Llama-7B-like attention projection n = m = 4096, N = 262144 bf16 samples,
+8 iterations per fit.  The inputs (4.3 GB) are larger than L2 (129 MB), so no
+flush is needed between steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With N > 1 (torchrun, one rank per GPU) every rank fits its own layer (independent
+problems, weak scaling, no collective in the data path); rank 0 prints the line.
+--impl reference times the fp64 CPU oracle on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+import synth  # noqa: E402
+
+METRIC = ("flip-flop iterations/s and weighted-Gram TFLOP/s (% of GB300 bf16 peak) per "
+          "layer shape")
+UNIT = "iterations/s"
+DEFAULT_WORKLOAD = "llama7b_attn_4096"
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
+    p.add_argument("--seed", type=int, default=0)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    return p.parse_args()
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, \
+            "fallback"
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ["clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.active",
+              "clocks_event_reasons.hw_slowdown", "clocks_event_reasons.hw_thermal_slowdown",
+              "clocks_event_reasons.sw_thermal_slowdown", "clocks_event_reasons.sw_power_cap"]
+
+    def __init__(self, device_index: int):
+        self.proc = None
+        try:
+            uuid = str(torch.cuda.get_device_properties(device_index).uuid)
+            sel = uuid if uuid.startswith("GPU-") else f"GPU-{uuid}"
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={','.join(self.FIELDS)}",
+                 "--format=csv,noheader,nounits", "-lms", "200", "-i", sel],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            return None
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < len(self.FIELDS):
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx = float(parts[1])
+            except ValueError:
+                continue
+            for nm, val in zip(names, parts[4:8]):
+                if val.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# ---------------------------------------------------------------------------
+# the fp64 CPU oracle on a bounded sample (reported baseline / reference arm)
+# ---------------------------------------------------------------------------
+def oracle_iteration_seconds(wl, X, G, n_sample: int):
+    """Seconds of one oracle flip-flop iteration at the workload's full N, from a
+    timed iteration on the first n_sample samples: the N-independent part (two
+    Cholesky factorisations) is timed on its own and not scaled; the rest is
+    linear in N and scaled by N / n_sample."""
+    import numpy as np
+
+    import oracle
+
+    Xs = oracle.as_f64(X[:n_sample])
+    Gs = oracle.as_f64(G[:n_sample])
+    t0 = time.perf_counter()
+    oracle.flipflop_fit(Xs, Gs, iters=1)
+    t_iter = time.perf_counter() - t0
+    A = np.eye(wl.n) + 0.0
+    B = np.eye(wl.m) + 0.0
+    t0 = time.perf_counter()
+    oracle.cholesky(A)
+    oracle.cholesky(B)
+    t_chol = time.perf_counter() - t0
+    lin = max(t_iter - t_chol, 0.0)
+    return t_chol + lin * (wl.N / n_sample), t_iter
+
+
+def oracle_sample_size(wl) -> int:
+    # about 1e12 fp64 flops per sampled iteration (a few seconds on a multi-core host)
+    per_sample = 4.0 * (wl.n ** 2 + wl.m ** 2)
+    return int(max(1024, min(wl.N, 1.0e12 / per_sample)))
+
+
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if rank != 0:
+        return 0
+    wl = synth.WORKLOADS[args.workload]
+    ns = oracle_sample_size(wl)
+    X, G = synth.rank_one_samples(wl, seed=args.seed, device="cpu", N=ns)
+    full = []
+    for i in range(args.warmup + args.steps):
+        t_full, _ = oracle_iteration_seconds(wl, X, G, ns)
+        if i >= args.warmup:
+            full.append(t_full)
+    t = statistics.mean(full)
+    value = 1.0 / t
+    sample = (f"one fp64 oracle iteration per step on the first {ns} of N={wl.N} samples "
+              f"(n={wl.n}, m={wl.m}); Cholesky part timed unscaled, the rest scaled by N/{ns}")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": t * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": wl.name, "N": wl.N, "n": wl.n, "m": wl.m,
+                   "iters_per_step": 1},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+def run_ours(args):
+    import paper_2609_14706_gb300 as ffh
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist_mod
+
+        dist_mod.init_process_group("nccl")
+        dist = dist_mod
+    wl = synth.WORKLOADS[args.workload]
+    if wl.kind != "rank_one":
+        raise SystemExit("bench.py times the rank-one fit")
+    iters = wl.iters
+    # each rank fits its own layer (independent problems)
+    X, G = synth.rank_one_samples(wl, seed=args.seed + rank, device="cuda")
+    N, n, m = wl.N, wl.n, wl.m
+    A = torch.empty(n, n, dtype=torch.float32, device="cuda")
+    B = torch.empty(m, m, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+    h = ffh.Handle(dtype=wl.dtype, profile=True, stream=stream)
+    for _ in range(max(args.warmup, 3)):
+        h.fit(X, G, iters, 0.0, A, B)
+    torch.cuda.synchronize()
+    h.timings(reset=True)
+    launches0 = h.timings()["kernel_launches"]
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    barrier()
+    clocks = ClockSampler(local)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        h.fit(X, G, iters, 0.0, A, B)
+    e1.record(stream)
+    barrier()
+    clk = clocks.stop()
+    elapsed_ms = e0.elapsed_time(e1)
+    tim = h.timings()
+    launches = tim["kernel_launches"] - launches0
+    if dist is not None:
+        t = torch.tensor([elapsed_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    value = world * args.steps * iters / (elapsed_ms / 1e3)
+
+    # ---- end to end through the C ABI with host buffers
+    e2e = None
+    if not args.no_e2e:
+        Xh = X.cpu().pin_memory()
+        Gh = G.cpu().pin_memory()
+        Ah = torch.empty(n, n, dtype=torch.float32).pin_memory()
+        Bh = torch.empty(m, m, dtype=torch.float32).pin_memory()
+        h2 = ffh.Handle(dtype=wl.dtype, stream=stream)
+        h2.fit(Xh, Gh, iters, 0.0, Ah, Bh)
+        barrier()
+        t0 = time.perf_counter()
+        f0 = torch.cuda.Event(enable_timing=True)
+        f1 = torch.cuda.Event(enable_timing=True)
+        f0.record(stream)
+        for _ in range(args.steps):
+            h2.fit(Xh, Gh, iters, 0.0, Ah, Bh)
+        f1.record(stream)
+        barrier()
+        wall_ms = (time.perf_counter() - t0) * 1e3
+        e2e_ms = max(f0.elapsed_time(f1), wall_ms)
+        if dist is not None:
+            t = torch.tensor([e2e_ms], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_ms = float(t.item())
+        h2.close()
+        e2e = {"value": world * args.steps * iters / (e2e_ms / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": Xh.numel() * Xh.element_size() + Gh.numel() * Gh.element_size(),
+               "d2h_bytes_per_step": (n * n + m * m) * 4}
+        del Xh, Gh
+
+    # ---- roofline of the dominant kernel (weighted Gram), measured live above
+    peaks, peak_kind = measured_peaks()
+    gram_flops_step = iters * (ffh.gram_flops(N, n) + ffh.gram_flops(N, m))
+    gram_tflops = (gram_flops_step * args.steps) / (tim["gram_ms"] / 1e3) / 1e12
+    peak = float(peaks.get("bf16_tflops_sustained", peaks.get("bf16_tflops")))
+    qform_flops_step = iters * (ffh.qform_flops(N, n) + ffh.qform_flops(N, m))
+    qform_tflops = (qform_flops_step * args.steps) / (tim["qform_ms"] / 1e3) / 1e12
+    roofline = {"bound": "tensor", "kernel": "k_gram_tc (weighted Gram)",
+                "achieved": gram_tflops, "peak": peak, "unit": "TFLOP/s",
+                "frac": gram_tflops / peak, "traffic": None,
+                "peak_source": f"{peak_kind} bf16 dense, sustained (kernel timed inside a long step)",
+                "flops_per_launch": (ffh.gram_flops(N, n) + ffh.gram_flops(N, m)) / 2,
+                "avg_launch_ms": tim["gram_ms"] / max(1, tim["gram_launches"])}
+    kernels = {
+        "gram_ms_per_step": tim["gram_ms"] / args.steps,
+        "qform_ms_per_step": tim["qform_ms"] / args.steps,
+        "chol_inv_ms_per_step": tim["chol_ms"] / args.steps,
+        "qform_tflops": qform_tflops,
+        "gram_frac_of_burst_peak": gram_tflops / float(peaks.get("bf16_tflops")),
+    }
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        ns = oracle_sample_size(wl)
+        t_full, t_sample = oracle_iteration_seconds(wl, X[:ns].cpu(), G[:ns].cpu(), ns)
+        cpu = {"value": 1.0 / t_full, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
+               "sample": (f"one fp64 oracle iteration on the first {ns} of N={N} samples "
+                          f"({t_sample:.1f} s); Cholesky part unscaled, rest scaled by N/{ns}")}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32",
+        "data": "synthetic",
+        "config": {"workload": wl.name, "N": N, "n": n, "m": m, "iters_per_step": iters,
+                   "parallelism": f"replicas{world}" if world > 1 else "single",
+                   "l2": "inputs (%.1f GB) exceed L2 (129 MB); no flush" %
+                         (wl.sample_bytes() / 1e9)},
+        "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e,
+        "gpu_launches": int(launches), "clocks": clk,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    h.close()
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

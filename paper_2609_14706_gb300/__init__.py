@@ -34,7 +34,15 @@ class ffh_options(ctypes.Structure):
     _fields_ = [("dtype", ctypes.c_int32), ("damping", ctypes.c_float),
                 ("variant", ctypes.c_int32), ("init_A", ctypes.c_void_p),
                 ("final_loglik", ctypes.c_int32), ("kernel", ctypes.c_int32),
-                ("fault", ctypes.c_int32), ("reserved", ctypes.c_int32 * 5)]
+                ("fault", ctypes.c_int32), ("profile", ctypes.c_int32),
+                ("reserved", ctypes.c_int32 * 4)]
+
+
+class ffh_timings(ctypes.Structure):
+    _fields_ = [("gram_ms", ctypes.c_double), ("gram_launches", ctypes.c_int64),
+                ("qform_ms", ctypes.c_double), ("qform_launches", ctypes.c_int64),
+                ("chol_ms", ctypes.c_double), ("chol_calls", ctypes.c_int64),
+                ("kernel_launches", ctypes.c_int64)]
 
 
 class FFHError(RuntimeError):
@@ -72,6 +80,7 @@ def load_library(path: Optional[str] = None):
         "ffh_weighted_gram": ([vp, vp, vp, i64, i64, f32, vp], ctypes.c_int),
         "ffh_quad_form": ([vp, vp, vp, i64, i64, vp], ctypes.c_int),
         "ffh_cholesky": ([vp, vp, i64, vp, vp, pd], ctypes.c_int),
+        "ffh_get_timings": ([vp, ctypes.POINTER(ffh_timings), i32], ctypes.c_int),
     }
     for name, (args, res) in sigs.items():
         fn = getattr(lib, name)
@@ -112,7 +121,8 @@ class Handle:
 
     def __init__(self, dtype="bf16", damping: float = 0.0, variant: str = "flipflop",
                  init_A: Optional[torch.Tensor] = None, final_loglik: bool = False,
-                 kernel: str = "tc", fault: int = 0, stream: Optional[torch.cuda.Stream] = None):
+                 kernel: str = "tc", fault: int = 0, profile: bool = False,
+                 stream: Optional[torch.cuda.Stream] = None):
         self._lib = load_library()
         self._keep = []
         self.opts = ffh_options()
@@ -126,6 +136,7 @@ class Handle:
         self.opts.final_loglik = int(bool(final_loglik))
         self.opts.kernel = {"tc": 0, "simt": 1}[kernel]
         self.opts.fault = int(fault)
+        self.opts.profile = int(bool(profile))
         self.stream = stream if stream is not None else torch.cuda.current_stream()
         self._h = ctypes.c_void_p()
         code = self._lib.ffh_create(ctypes.byref(self._h), ctypes.byref(self.opts),
@@ -205,6 +216,13 @@ class Handle:
         k = min(ntr.value, capacity)
         return {"iters_done": it.value, "delta": delta.value, "loglik": list(ll[:k]),
                 "mean_qr": list(mqr[:k])}
+
+    def timings(self, reset: bool = False) -> dict:
+        """ffh_get_timings: kernel times accumulated while profile=True."""
+        t = ffh_timings()
+        code = self._lib.ffh_get_timings(self._h, ctypes.byref(t), int(bool(reset)))
+        _check(self._lib, self._h, code, "ffh_get_timings")
+        return {f: getattr(t, f) for f, _ in ffh_timings._fields_}
 
     # -- single steps --
     def weighted_gram(self, V: torch.Tensor, w: Optional[torch.Tensor], scale: float = 1.0,
