@@ -185,6 +185,26 @@ ffh_status ffh_quad_form(ffh_t h, const void* V, const float* Linv, int64_t N, i
 ffh_status ffh_cholesky(ffh_t h, const float* F, int64_t d, float* L_out, float* Linv_out,
                         double* logdet);
 
+/* Weighted Gram that allocates no device memory.  The paper has no counterpart: this
+ * entry point exists for callers that cannot call cudaMalloc -- code running inside a
+ * framework that owns all device memory (a pre-reserved pool, an inference-engine
+ * plugin) or a latency-critical path where an allocation would synchronise the device.
+ *   Computes the same C = scale * V^T diag(w) V as ffh_weighted_gram (bf16 V, N x d,
+ *   d a multiple of 8; w N fp32 or NULL; C_out d x d fp32), with no handle.
+ *   V, w, C_out: device pointers owned by the caller.  cuda_stream: cudaStream_t.
+ *   errbuf / errbuf_len: optional caller buffer that receives a message.
+ * Working memory comes from one static device array of 64 MiB that the library holds
+ * on every GPU where it is loaded, until the process exits; N, d whose working memory
+ * does not fit (roughly d > 5000) are rejected with FFH_ERR_INVALID_ARG before any
+ * GPU work.  The first call on a device looks up the array's address (set-up); make
+ * that first call before any stream capture.  All calls share the array and it keeps
+ * the last call's contents (this call clears what must start at zero): calls whose
+ * work overlaps on the GPU race and must be serialised by the caller.  The call
+ * synchronises `cuda_stream` once to read the status word. */
+ffh_status ffh_weighted_gram_static(const void* V, const float* w, int64_t N, int64_t d,
+                                    float scale, float* C_out, void* cuda_stream,
+                                    char* errbuf, int32_t errbuf_len);
+
 #ifdef __cplusplus
 }
 #endif

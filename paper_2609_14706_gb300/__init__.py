@@ -81,6 +81,8 @@ def load_library(path: Optional[str] = None):
         "ffh_quad_form": ([vp, vp, vp, i64, i64, vp], ctypes.c_int),
         "ffh_cholesky": ([vp, vp, i64, vp, vp, pd], ctypes.c_int),
         "ffh_get_timings": ([vp, ctypes.POINTER(ffh_timings), i32], ctypes.c_int),
+        "ffh_weighted_gram_static": ([vp, vp, i64, i64, f32, vp, vp, ctypes.c_char_p, i32],
+                                     ctypes.c_int),
     }
     for name, (args, res) in sigs.items():
         fn = getattr(lib, name)
@@ -263,6 +265,29 @@ class Handle:
         return L, Li, ld.value
 
 
+def weighted_gram_static(V: torch.Tensor, w: Optional[torch.Tensor], scale: float = 1.0,
+                         C_out: Optional[torch.Tensor] = None,
+                         stream: Optional[torch.cuda.Stream] = None) -> torch.Tensor:
+    """ffh_weighted_gram_static: scale * V^T diag(w) V with no device allocation by the
+    library (bf16 V on the device; see include/ffh.h for the limits)."""
+    lib = load_library()
+    if V.dtype != torch.bfloat16:
+        raise TypeError("V must be bfloat16")
+    V = V.contiguous()
+    N, d = V.shape
+    if w is not None:
+        w = w.to(torch.float32).contiguous()
+    if C_out is None:
+        C_out = torch.empty(d, d, dtype=torch.float32, device=V.device)
+    stream = stream if stream is not None else torch.cuda.current_stream()
+    buf = ctypes.create_string_buffer(256)
+    code = lib.ffh_weighted_gram_static(_ptr(V), _ptr(w), N, d, float(scale), _ptr(C_out),
+                                        ctypes.c_void_p(stream.cuda_stream), buf, 256)
+    if code != 0:
+        raise FFHError(code, "ffh_weighted_gram_static", buf.value.decode())
+    return C_out
+
+
 def fit(X: torch.Tensor, G: torch.Tensor, iters: int, tol: float = 0.0, **options):
     """One-shot ffh_fit with a temporary handle; returns (A, B, stats)."""
     dtype = "bf16" if X.dtype == torch.bfloat16 else "f32"
@@ -292,5 +317,5 @@ def iteration_flops(N: int, n: int, m: int) -> float:
     return gram_flops(N, n) + gram_flops(N, m) + qform_flops(N, n) + qform_flops(N, m)
 
 
-__all__ = ["Handle", "FFHError", "fit", "fit_matrix", "load_library", "header_symbols",
+__all__ = ["Handle", "FFHError", "fit", "fit_matrix", "weighted_gram_static", "load_library", "header_symbols",
            "gram_flops", "qform_flops", "iteration_flops", "ffh_options"]
