@@ -323,7 +323,10 @@ ffh_status qform(ffh_t h, const Staged& V, int64_t N, int64_t d, const float* Li
 ffh_status chol(ffh_t h, const float* F, int64_t d, float* L, float* Linv, float* work, float* DI,
                 DevStatus* st, int fault) {
   cudaEvent_t t0 = prof_begin(h);
-  CK(launch_cholesky(F, d, d, L, Linv, work, DI, st, fault, h->stream));
+  if (h->opt.kernel == 1)
+    CK(launch_cholesky(F, d, d, L, Linv, work, DI, st, fault, h->stream));
+  else
+    CK(launch_cholesky_tc(F, d, d, L, Linv, work, st, fault, h->stream));
   prof_end(h, PROF_CHOL, t0);
   return FFH_OK;
 }
@@ -333,7 +336,7 @@ ffh_status setup_tables(ffh_t h, int64_t N, int64_t d, GramTables* gt, int2* til
   gt->plan = gram_plan(N, d, num_sms());
   gt->tiles = tiles_dev;
   gt->lut = lut_dev;
-  const int64_t nbm = (d + 127) / 128, nbn = (d + 255) / 256;
+  const int64_t nbm = (d + kGramBM - 1) / kGramBM, nbn = (d + kGramBN - 1) / kGramBN;
   std::vector<int2> tiles((size_t)(nbm * nbn));
   std::vector<int> lut((size_t)(nbm * nbn));
   int T = 0;
@@ -394,7 +397,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
     *L = c.take<float>((size_t)D * D);
     *Linv = c.take<float>((size_t)D * D);
     *Mb = c.take<__nv_bfloat16>((size_t)D * pad8(D));
-    *work = c.take<float>(cholesky_work_floats(D));
+    *work = c.take<float>(std::max(cholesky_work_floats(D), cholesky_tc_work_bytes(D) / 4 + 1));
     *DI = c.take<float>((size_t)nt * 64 * 64);
     *tn = c.take<int2>(gram_tile_table_bytes(n) / sizeof(int2) + 1);
     *ln = c.take<int>(gram_tile_table_bytes(n) / sizeof(int) + 1);
@@ -696,7 +699,7 @@ extern "C" ffh_status ffh_cholesky(ffh_t h, const float* F, int64_t d, float* L_
     *st = c.take<DevStatus>(1);
     *L = L_out ? nullptr : c.take<float>((size_t)d * d);
     *Li = c.take<float>((size_t)d * d);
-    *work = c.take<float>(cholesky_work_floats(d));
+    *work = c.take<float>(std::max(cholesky_work_floats(d), cholesky_tc_work_bytes(d) / 4 + 1));
     *DI = c.take<float>((size_t)nt * 64 * 64);
   };
   DevStatus* st;

@@ -54,10 +54,15 @@ void note_launches(int k);
 long long launches_so_far();
 
 // tensor-core kernels (kernels_tc.cu)
+// weighted-Gram output tile (rows x cols); a tile is computed iff it meets the lower
+// triangle: tile_col * kGramBN <= tile_row * kGramBM + kGramBM - 1
+constexpr int kGramBM = 256;
+constexpr int kGramBN = 256;
+constexpr int kGramBK = 32;   // samples per pipeline stage (weights padded to this)
 struct GramPlan {
   int T;        // lower-triangle output tiles
   int S;        // K splits
-  int KB;       // 64-sample blocks
+  int KB;       // kGramBK-sample blocks
   int units;    // T * S
   int grid;     // persistent CTAs
 };
@@ -92,6 +97,10 @@ cudaError_t launch_cholesky(const float* F, int64_t d, int64_t ldf, float* L, fl
                             float* work, float* diag_inv, DevStatus* st, int fault,
                             cudaStream_t s);
 size_t cholesky_work_floats(int64_t d);
+// tensor-core Cholesky + inverse (kernels_chol.cu); `work` of cholesky_tc_work_bytes(d)
+cudaError_t launch_cholesky_tc(const float* F, int64_t d, int64_t ldf, float* L, float* Linv,
+                               void* work, DevStatus* st, int fault, cudaStream_t s);
+size_t cholesky_tc_work_bytes(int64_t d);
 cudaError_t launch_fill_identity(float* F, int64_t d, int64_t ld, cudaStream_t s);
 cudaError_t launch_damp(float* F, int64_t d, int64_t ld, float lambda, DevStatus* st,
                         cudaStream_t s);

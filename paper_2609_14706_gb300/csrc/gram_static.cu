@@ -50,7 +50,7 @@ __global__ void k_static_tiles(int64_t d, int nbm, int nbn, int2* tiles, int* lu
   int T = 0;
   for (int ti = 0; ti < nbm; ++ti)
     for (int tj = 0; tj < nbn; ++tj) {
-      const bool need = (int64_t)tj * 256 <= (int64_t)ti * 128 + 127;
+      const bool need = (int64_t)tj * kGramBN <= (int64_t)ti * kGramBM + kGramBM - 1;
       lut[ti * nbn + tj] = need ? T : -1;
       if (need) tiles[T++] = make_int2(ti, tj);
     }
@@ -99,7 +99,7 @@ extern "C" ffh_status ffh_weighted_gram_static(const void* V, const float* w, in
     return FFH_ERR_UNSUPPORTED;
   }
   // the working-memory layout for this call; reject what does not fit
-  const int64_t nbm = (d + 127) / 128, nbn = (d + 255) / 256;
+  const int64_t nbm = (d + kGramBM - 1) / kGramBM, nbn = (d + kGramBN - 1) / kGramBN;
   const int64_t Npad = (N + 63) / 64 * 64 + 64;
   GramPlan plan = gram_plan(N, d, num_sms());
   const size_t fixed = align256(sizeof(DevStatus)) + align256(sizeof(int2) * nbm * nbn) +

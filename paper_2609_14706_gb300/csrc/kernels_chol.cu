@@ -1,0 +1,637 @@
+// Tensor-core Cholesky factor and triangular inverse of the d x d factors A, B.
+//
+// Blocked right-looking Cholesky with 128-wide panels (Section 2 notation: L lower,
+// L L^T = F):
+//   * k_chol_leaf  factors the 128 x 128 diagonal block in shared memory (one CTA) and,
+//                  in the same column sweep, its inverse M11 = L11^-1 (each elimination
+//                  step applied to the identity as well);
+//   * the panel below, L21 = A21 M11^T, and the trailing update A22 -= L21 L21^T are
+//     tcgen05 GEMMs (k_gemm_tc);
+// then M = L^-1 by recursive doubling over the diagonal-block inverses:
+//   [[L11, 0], [L21, L22]]^-1 = [[M11, 0], [-M22 (L21 M11), M22]].
+//
+// fp32 operands enter the bf16 tensor cores as a hi/lo split (x = hi + lo, both bf16):
+// a b ~ hi_a hi_b + hi_a lo_b + lo_a hi_b, accumulated in fp32 (relative error of a
+// product ~2^-16).  The split is laid out as [hi | lo] along K, so the three products
+// are one GEMM over three K segments.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+
+#include "ffh_internal.cuh"
+#include "tc_ptx.cuh"
+
+namespace ffh {
+
+using namespace ptx;
+
+static constexpr uint64_t kGemmWaitNs = 4000000000ull;
+
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn_chol() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+static bool map_bf16_kmajor(CUtensorMap* m, const void* base, uint64_t k_extent, uint64_t rows,
+                            uint64_t pitch_elems, uint32_t box_rows) {
+  auto fn = encode_fn_chol();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {k_extent, rows};
+  cuuint64_t strides[1] = {pitch_elems * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// ===========================================================================
+// TN GEMM on tcgen05:  C[z] = alpha * A'[z] B'[z]^T + beta * C[z]
+//   A'[z]: M x K' bf16 rows (K-major), B'[z]: N x K' bf16 rows (K-major); both are the
+//   packed rows z*rows_pad .. of one 2-D buffer.  K' is a list of up to three 64-aligned
+//   segments (x offsets per operand), each kseg wide.
+//   C: fp32 row-major, element (r, c) of batch z at C + z*strideC + r*ldc + c.
+// ===========================================================================
+namespace gt {
+constexpr int BM = 128, BN = 128, BK = 64, STAGES = 4;
+constexpr int A_BYTES = BM * BK * 2, B_BYTES = BN * BK * 2;
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
+constexpr uint32_t TMEM_COLS = 128;
+}  // namespace gt
+
+struct GemmTcArgs {
+  float* C;
+  int64_t ldc, strideC;
+  int M, N;                 // valid rows / cols of C per batch
+  int a_rows_pad, b_rows_pad;  // packed rows per batch in the A' / B' buffers
+  int nseg, kseg_blocks;    // segments, 64-blocks per segment
+  int a_off[3], b_off[3];   // x offsets (elements) of the segments
+  float alpha, beta;
+  int lower_only;           // skip tiles strictly above the diagonal
+  __nv_bfloat16* split_out; // optional: also write the bf16 hi/lo split of the result,
+  int split_kpad;           //   row r of batch z at (z*M_pad + r) * 2*split_kpad
+  int split_rows_pad;
+  DevStatus* st;
+};
+
+__global__ void __launch_bounds__(256, 1)
+    k_gemm_tc(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
+              const GemmTcArgs a) {
+  using namespace gt;
+  const int tn = blockIdx.x, tm = blockIdx.y, z = blockIdx.z;
+  const int row0 = tm * BM, col0 = tn * BN;
+  if (a.lower_only && col0 > row0 + BM - 1) return;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + STAGES;
+  uint64_t* accf = bars + 2 * STAGES;
+  uint64_t* drain = accf + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  volatile int* skip_flag = abort_flag + 1;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    *skip_flag = *reinterpret_cast<volatile int*>(&a.st->abort_all);
+    *abort_flag = 0;
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(accf, 1);
+    mbar_init(drain, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (*skip_flag) return;
+  if (warp == 2) {
+    tmem_alloc(tmem_slot, TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const int nk = a.nseg * a.kseg_blocks;
+  const int arow = z * a.a_rows_pad + row0, brow = z * a.b_rows_pad + col0;
+
+  if (warp == 0 && lane == 0) {
+    bool ok = true;
+    int it = 0;
+    for (; it < nk; ++it) {
+      const int s = it % STAGES;
+      const uint32_t ph = (it / STAGES) & 1;
+      if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, kGemmWaitNs)) {
+        ok = false;
+        break;
+      }
+      const int seg = it / a.kseg_blocks, kb = it - seg * a.kseg_blocks;
+      mbar_arrive_expect_tx(&full[s], STAGE_BYTES);
+      uint8_t* sa = smem + s * STAGE_BYTES;
+      tma_load_2d(sa, &amap, &full[s], a.a_off[seg] + kb * BK, arow);
+      tma_load_2d(sa + A_BYTES, &bmap, &full[s], a.b_off[seg] + kb * BK, brow);
+    }
+    if (!ok) {
+      *abort_flag = 1;
+      raise_error(a.st, FFH_ERR_TIMEOUT, 21);
+    }
+    const int first = it > STAGES ? it - STAGES : 0;
+    for (int j = first; j < it; ++j) {
+      volatile int never = 0;
+      mbar_wait(&full[j % STAGES], (j / STAGES) & 1, &never, kGemmWaitNs);
+    }
+  } else if (warp == 1 && lane == 0) {
+    constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, false, false);
+    bool ok = true;
+    for (int it = 0; it < nk; ++it) {
+      const int s = it % STAGES;
+      const uint32_t ph = (it / STAGES) & 1;
+      if (!mbar_wait(&full[s], ph, abort_flag, kGemmWaitNs)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t sa = smem_u32(smem + s * STAGE_BYTES), sb = sa + A_BYTES;
+#pragma unroll
+      for (int k = 0; k < BK / 16; ++k)
+        mma_bf16(tmem, sw128_desc(sa + k * 32, 16, 1024), sw128_desc(sb + k * 32, 16, 1024),
+                 idesc, (it > 0 || k > 0) ? 1u : 0u);
+      mma_commit(&empty[s]);
+    }
+    if (ok) {
+      mma_commit(accf);
+    } else {
+      *abort_flag = 1;
+      raise_error(a.st, FFH_ERR_TIMEOUT, 22);
+    }
+    mma_commit(drain);
+    volatile int never = 0;
+    mbar_wait(drain, 0, &never, kGemmWaitNs);
+  } else if (warp >= 4) {
+    const int wq = warp - 4;
+    if (mbar_wait(accf, 0, abort_flag, kGemmWaitNs)) {
+      tc_fence_after();
+      // every MMA has completed (accf), so the stage buffers are free: each warp
+      // transposes its 32 x 32 chunks through shared memory and stores rows
+      // contiguously across lanes.
+      float* tb = reinterpret_cast<float*>(smem) + wq * 32 * 33;
+      const int rbase = row0 + wq * 32;
+#pragma unroll 1
+      for (int cb = 0; cb < BN / 32; ++cb) {
+        float v[32];
+        tmem_ld32(tmem + ((uint32_t)(wq * 32) << 16) + cb * 32, v);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) tb[lane * 33 + j] = v[j];
+        __syncwarp();
+        const int c = col0 + cb * 32 + lane;
+        float* cbase = a.C + (int64_t)z * a.strideC + (int64_t)rbase * a.ldc + c;
+        // all loads of C first (independent, in flight together), then the stores
+        float prev[32];
+        if (a.beta != 0.f) {
+#pragma unroll
+          for (int rr = 0; rr < 32; ++rr)
+            prev[rr] = (rbase + rr < a.M && c < a.N) ? cbase[(int64_t)rr * a.ldc] : 0.f;
+        }
+#pragma unroll
+        for (int rr = 0; rr < 32; ++rr) {
+          const int r = rbase + rr;
+          if (r < a.M && c < a.N) {
+            const float o = a.alpha * tb[rr * 33 + lane];
+            const float res = a.beta == 0.f ? o : fmaf(a.beta, prev[rr], o);
+            cbase[(int64_t)rr * a.ldc] = res;
+            if (a.split_out) {
+              __nv_bfloat16* srow =
+                  a.split_out + ((int64_t)z * a.split_rows_pad + r) * 2 * a.split_kpad;
+              const __nv_bfloat16 hi = __float2bfloat16_rn(res);
+              srow[c] = hi;
+              srow[a.split_kpad + c] = __float2bfloat16_rn(res - __bfloat162float(hi));
+            }
+          }
+        }
+        __syncwarp();
+      }
+      tc_fence_before();
+    } else {
+      *abort_flag = 1;
+      raise_error(a.st, FFH_ERR_TIMEOUT, 23);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+// A bf16 hi/lo split buffer: rows x [hi (kpad) | lo (kpad)], pitch 2*kpad, kpad = 64-aligned.
+struct Split {
+  __nv_bfloat16* p;
+  int rows_pad;   // packed rows per batch (>= valid rows; rows beyond are masked outputs)
+  int kpad;       // 64-aligned K extent of one half
+  int batch;
+};
+
+static cudaError_t gemm_tc(const Split& A, const Split& B, int nseg, const int a_seg[3],
+                           const int b_seg[3], int kseg, float* C, int64_t ldc, int64_t strideC,
+                           int M, int N, float alpha, float beta, bool lower_only, int batch,
+                           DevStatus* st, cudaStream_t s, const Split* out_split = nullptr) {
+  if (M <= 0 || N <= 0 || batch <= 0) return cudaSuccess;
+  CUtensorMap am, bm;
+  if (!map_bf16_kmajor(&am, A.p, (uint64_t)2 * A.kpad, (uint64_t)A.rows_pad * A.batch,
+                       (uint64_t)2 * A.kpad, gt::BM))
+    return cudaErrorInvalidValue;
+  if (!map_bf16_kmajor(&bm, B.p, (uint64_t)2 * B.kpad, (uint64_t)B.rows_pad * B.batch,
+                       (uint64_t)2 * B.kpad, gt::BN))
+    return cudaErrorInvalidValue;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         gt::SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  GemmTcArgs g{};
+  g.C = C;
+  g.ldc = ldc;
+  g.strideC = strideC;
+  g.M = M;
+  g.N = N;
+  g.a_rows_pad = A.rows_pad;
+  g.b_rows_pad = B.rows_pad;
+  g.nseg = nseg;
+  g.kseg_blocks = (kseg + 63) / 64;
+  for (int i = 0; i < 3; ++i) {
+    g.a_off[i] = a_seg[i];
+    g.b_off[i] = b_seg[i];
+  }
+  g.alpha = alpha;
+  g.beta = beta;
+  g.lower_only = lower_only ? 1 : 0;
+  g.split_out = out_split ? out_split->p : nullptr;
+  g.split_kpad = out_split ? out_split->kpad : 0;
+  g.split_rows_pad = out_split ? out_split->rows_pad : 0;
+  g.st = st;
+  dim3 grid((N + gt::BN - 1) / gt::BN, (M + gt::BM - 1) / gt::BM, batch);
+  k_gemm_tc<<<grid, 256, gt::SMEM_BYTES, s>>>(am, bm, g);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// fp32 -> bf16 hi/lo split, optionally transposed, batched:
+//   batch z, row r < rows, col c < cols of the source view
+//     src[z*src_stride + r*lds + c]          (trans = 0)
+//     src[z*src_stride + c*lds + r]          (trans = 1: output row r = source column r)
+//   dst[(z*rows_pad + r)*2kpad + c] = hi, [... + kpad + c] = lo; zero elsewhere up to
+//   rows_pad x 2kpad.
+// ---------------------------------------------------------------------------
+__global__ void k_split_hilo(const float* __restrict__ src, int64_t lds, int64_t src_stride,
+                             int rows, int cols, int trans, __nv_bfloat16* __restrict__ dst,
+                             int rows_pad, int kpad, int batch) {
+  const int64_t per = (int64_t)rows_pad * kpad;
+  const int64_t total = per * batch;
+  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+       idx += (int64_t)gridDim.x * blockDim.x) {
+    const int z = (int)(idx / per);
+    const int64_t rem = idx - (int64_t)z * per;
+    const int r = (int)(rem / kpad), c = (int)(rem - (int64_t)r * kpad);
+    float x = 0.f;
+    if (r < rows && c < cols) {
+      const float* sz = src + (int64_t)z * src_stride;
+      x = trans ? sz[(int64_t)c * lds + r] : sz[(int64_t)r * lds + c];
+    }
+    const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+    const __nv_bfloat16 lo = __float2bfloat16_rn(x - __bfloat162float(hi));
+    __nv_bfloat16* drow = dst + ((int64_t)z * rows_pad + r) * (2 * (int64_t)kpad);
+    drow[c] = hi;
+    drow[kpad + c] = lo;
+  }
+}
+
+static cudaError_t split(const float* src, int64_t lds, int64_t src_stride, int rows, int cols,
+                         bool trans, const Split& d, cudaStream_t s) {
+  const int64_t total = (int64_t)d.rows_pad * d.kpad * d.batch;
+  if (total == 0) return cudaSuccess;
+  const int64_t blocks = std::min<int64_t>((total + 255) / 256, (int64_t)num_sms() * 16);
+  k_split_hilo<<<(unsigned)blocks, 256, 0, s>>>(src, lds, src_stride, rows, cols, trans ? 1 : 0,
+                                                d.p, d.rows_pad, d.kpad, d.batch);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// 128 x 128 diagonal block: Cholesky factor L11 and inverse M11 = L11^-1 in shared
+// memory, one CTA of 512 threads.
+//   Factorisation: four 32-column sub-panels.  Within a sub-panel, each pivot step j
+//   updates only the sub-panel's columns (j, c0+32) of the rows below (one column per
+//   lane, rows spread over the 16 warps); the scaling of column j by 1/sqrt(pivot) is
+//   deferred to step j+1, which neither reads nor writes column j, so each step costs
+//   one barrier.  The finished sub-panel then updates the trailing lower triangle as a
+//   rank-32 product (4 x 4 register blocks).
+//   Inverse: the four 32 x 32 diagonal blocks by forward substitution (one warp each,
+//   lane c computes column c), then off-diagonal blocks by doubling,
+//   [[L11,0],[L21,L22]]^-1 = [[M11,0],[-M22 (L21 M11), M22]].
+// Outputs: L11 and M11 (fp32) and the bf16 hi/lo split of M11 ([hi | lo] rows, pitch
+// 256), the B operand of the panel GEMM.
+// ---------------------------------------------------------------------------
+constexpr int LB = 128;
+constexpr int LP = LB + 1;  // padded pitch
+constexpr int LB_SMEM = (2 * LB * LP + 64 * 65) * 4 + 64;
+constexpr int LEAF_THREADS = 512;
+
+// C[r][c] (+)= sgn * sum_k A[r][k] B[k][c] on a 32 x 32 (or 64 x 64) block in shared
+// memory, with 4 x 4 register blocks; thread t of nthreads covers blocks t, t+nthreads.
+template <int S>
+__device__ __forceinline__ void smem_gemm(float* C, int ldc, const float* A, int lda,
+                                          const float* B, int ldb, int kbeg, int kend, float sgn,
+                                          bool accumulate, int t, int nthreads) {
+  constexpr int NB = S / 4;
+  for (int blk = t; blk < NB * NB; blk += nthreads) {
+    const int br = (blk / NB) * 4, bc = (blk % NB) * 4;
+    float acc[4][4] = {};
+    for (int k = kbeg; k < kend; ++k) {
+      float av[4], bv[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) av[i] = A[(br + i) * lda + k];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) bv[j] = B[k * ldb + bc + j];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        float* cp = C + (br + i) * ldc + bc + j;
+        *cp = accumulate ? fmaf(sgn, acc[i][j], *cp) : sgn * acc[i][j];
+      }
+  }
+}
+
+__global__ void __launch_bounds__(LEAF_THREADS) k_chol_leaf(float* W, int64_t ldw, int64_t d,
+                                                            int64_t o, float* L, int64_t ldl,
+                                                            float* Minv, int64_t ldm,
+                                                            __nv_bfloat16* m11_split,
+                                                            DevStatus* st, int fault) {
+  extern __shared__ float sh[];
+  float* Ls = sh;             // [LB][LP]
+  float* Ms = sh + LB * LP;   // [LB][LP]
+  float* Ts = sh + 2 * LB * LP;  // [64][65] temporary
+  const int b = (int)((d - o) < LB ? (d - o) : LB);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  for (int idx = tid; idx < LB * LB / 4; idx += LEAF_THREADS) {
+    const int i = idx >> 5, j4 = (idx & 31) * 4;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (i < b) {
+      const float* src = W + (o + i) * ldw + o + j4;
+      if (j4 + 3 < b && (((uintptr_t)src) & 15) == 0) {
+        v = *reinterpret_cast<const float4*>(src);
+      } else {
+        if (j4 + 0 < b) v.x = src[0];
+        if (j4 + 1 < b) v.y = src[1];
+        if (j4 + 2 < b) v.z = src[2];
+        if (j4 + 3 < b) v.w = src[3];
+      }
+    }
+    const float vv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int j = j4 + e;
+      float x = (j <= i) ? vv[e] : 0.f;
+      if (i >= b || j >= b) x = (i == j) ? 1.f : 0.f;
+      Ls[i * LP + j] = x;
+      Ms[i * LP + j] = 0.f;
+    }
+  }
+  __syncthreads();
+  if (tid == 0 && fault == FFH_FAULT_BAD_PIVOT && o == 0) Ls[0] = __int_as_float(0x7fc00000);
+  __syncthreads();
+  float ld_acc = 0.f;
+  bool bad = false;
+  for (int q = 0; q < LB / 32; ++q) {
+    const int c0 = 32 * q;
+    const int x = c0 + lane;  // this lane's column of the sub-panel
+    float rinv_prev = 1.f, r_prev = 1.f;
+    for (int jj = 0; jj <= 32; ++jj) {
+      const int j = c0 + jj;
+      // deferred scaling of column j-1 (rows >= j) and its pivot
+      if (jj > 0) {
+        if (tid < LB - j)
+          Ls[(j + tid) * LP + j - 1] *= rinv_prev;
+        else if (tid == LB - j)
+          Ls[(j - 1) * LP + j - 1] = r_prev;
+      }
+      if (jj == 32) break;
+      float ajj = Ls[j * LP + j];
+      if (!(ajj > 0.f) || !isfinite(ajj)) {
+        if (tid == 0 && !bad) raise_error(st, FFH_ERR_NOT_SPD, (int)(o + j));
+        bad = true;
+        ajj = 1.f;
+      }
+      const float r = sqrtf(ajj);
+      const float rinv = 1.f / r;
+      if (tid == 0 && j < b) ld_acc += logf(r);
+      if (x > j) {
+        const float lxj = Ls[x * LP + j] * rinv;
+        for (int i = j + 1 + ((warp - (j + 1)) & 15); i < LB; i += 16)
+          if (x <= i) Ls[i * LP + x] = fmaf(-Ls[i * LP + j] * rinv, lxj, Ls[i * LP + x]);
+      }
+      rinv_prev = rinv;
+      r_prev = r;
+      __syncthreads();
+    }
+    __syncthreads();
+    // trailing rank-32 update of the lower triangle: A[r][c] -= sum_k L[r][c0+k] L[c][c0+k]
+    const int r0 = c0 + 32;
+    const int nb = (LB - r0) / 4;  // 4 x 4 blocks per side
+    for (int blk = tid; blk < nb * nb; blk += LEAF_THREADS) {
+      const int bi = blk / nb, bj = blk - bi * nb;
+      if (bj > bi) continue;
+      const int rr = r0 + 4 * bi, cc = r0 + 4 * bj;
+      float acc[4][4] = {};
+#pragma unroll 4
+      for (int k = 0; k < 32; ++k) {
+        float av[4], bv[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) av[i] = Ls[(rr + i) * LP + c0 + k];
+#pragma unroll
+        for (int jx = 0; jx < 4; ++jx) bv[jx] = Ls[(cc + jx) * LP + c0 + k];
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+          for (int jx = 0; jx < 4; ++jx) acc[i][jx] = fmaf(av[i], bv[jx], acc[i][jx]);
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int jx = 0; jx < 4; ++jx)
+          if (cc + jx <= rr + i) Ls[(rr + i) * LP + cc + jx] -= acc[i][jx];
+    }
+    __syncthreads();
+  }
+  // inverse of the four 32 x 32 diagonal blocks: warp q, lane c computes column c
+  if (warp < 4) {
+    const int c0 = 32 * warp, c = lane;
+    for (int i = 0; i < 32; ++i) {
+      float acc = (i == c) ? 1.f : 0.f;
+      if (i >= c) {
+        for (int k = c; k < i; ++k)
+          acc = fmaf(-Ls[(c0 + i) * LP + c0 + k], Ms[(c0 + k) * LP + c0 + c], acc);
+        Ms[(c0 + i) * LP + c0 + c] = acc / Ls[(c0 + i) * LP + c0 + i];
+      }
+    }
+  }
+  __syncthreads();
+  // doubling, h = 32: pairs (0,1) and (2,3); h = 64: pair (0,1)
+  {
+    // pair pr = tid / 256 (threads 0-255 take pair 0, 256-511 pair 1); T = L21 M11
+    // (32 x 32, pair pr in columns 32 pr .. of Ts), then M21 = -M22 T
+    const int pr = tid >> 8, tp = tid & 255, ob = 64 * pr;
+    smem_gemm<32>(Ts + pr * 32, 65, Ls + (ob + 32) * LP + ob, LP, Ms + ob * LP + ob, LP, 0, 32,
+                  1.f, false, tp, 256);
+    __syncthreads();
+    smem_gemm<32>(Ms + (ob + 32) * LP + ob, LP, Ms + (ob + 32) * LP + ob + 32, LP, Ts + pr * 32,
+                  65, 0, 32, -1.f, false, tp, 256);
+    __syncthreads();
+  }
+  smem_gemm<64>(Ts, 65, Ls + 64 * LP, LP, Ms, LP, 0, 64, 1.f, false, tid, LEAF_THREADS);
+  __syncthreads();
+  smem_gemm<64>(Ms + 64 * LP, LP, Ms + 64 * LP + 64, LP, Ts, 65, 0, 64, -1.f, false, tid,
+                LEAF_THREADS);
+  __syncthreads();
+  for (int idx = tid; idx < LB * LB; idx += LEAF_THREADS) {
+    const int i = idx >> 7, j = idx & 127;
+    const float mv = (j <= i) ? Ms[i * LP + j] : 0.f;
+    if (i < b && j < b) {
+      L[(o + i) * ldl + (o + j)] = (j <= i) ? Ls[i * LP + j] : 0.f;
+      Minv[(o + i) * ldm + (o + j)] = mv;
+    }
+    if (m11_split) {
+      const float xx = (i < b && j < b) ? mv : 0.f;
+      const __nv_bfloat16 hi = __float2bfloat16_rn(xx);
+      m11_split[i * 2 * LB + j] = hi;
+      m11_split[i * 2 * LB + LB + j] = __float2bfloat16_rn(xx - __bfloat162float(hi));
+    }
+  }
+  if (tid == 0) atomicAdd(&st->logdet, 2.0 * (double)ld_acc);
+}
+
+size_t cholesky_tc_work_bytes(int64_t d) {
+  const int64_t kmax = (d + 63) / 64 * 64;
+  const int64_t rows = (d + 127) / 128 * 128 + 128;
+  // W copy, T scratch, four split buffers (each <= rows x 2*kmax bf16)
+  return (size_t)d * d * 4 + (size_t)d * d * 4 + 4 * (size_t)rows * 2 * kmax * 2 + 4096;
+}
+
+// L (lower), Linv = L^-1 (lower); st->logdet += log|F|.  F is read, not modified.
+cudaError_t launch_cholesky_tc(const float* F, int64_t d, int64_t ldf, float* L, float* Linv,
+                               void* work, DevStatus* st, int fault, cudaStream_t s) {
+  cudaError_t e;
+  const int64_t kmax = (d + 63) / 64 * 64;
+  const int64_t rows_cap = (d + 127) / 128 * 128 + 128;
+  char* wp = static_cast<char*>(work);
+  float* W = reinterpret_cast<float*>(wp);
+  wp += (size_t)d * d * 4;
+  float* T = reinterpret_cast<float*>(wp);
+  wp += (size_t)d * d * 4;
+  __nv_bfloat16* sb[4];
+  for (int i = 0; i < 4; ++i) {
+    sb[i] = reinterpret_cast<__nv_bfloat16*>(wp);
+    wp += (size_t)rows_cap * 2 * kmax * 2;
+  }
+  static bool attr = false;
+  if (!attr) {
+    if ((e = cudaFuncSetAttribute(k_chol_leaf, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  LB_SMEM)) != cudaSuccess)
+      return e;
+    attr = true;
+  }
+  if ((e = cudaMemcpy2DAsync(W, d * 4, F, ldf * 4, d * 4, d, cudaMemcpyDeviceToDevice, s)) !=
+      cudaSuccess)
+    return e;
+  if ((e = cudaMemsetAsync(L, 0, (size_t)d * d * 4, s)) != cudaSuccess) return e;
+  if (Linv && (e = cudaMemsetAsync(Linv, 0, (size_t)d * d * 4, s)) != cudaSuccess) return e;
+  if ((e = cudaMemsetAsync(&st->logdet, 0, sizeof(double), s)) != cudaSuccess) return e;
+  float* Mdiag = Linv ? Linv : T;  // the diagonal-block inverses (T is free until the inverse)
+  const int np = (int)((d + LB - 1) / LB);
+  for (int p = 0; p < np; ++p) {
+    const int64_t o = (int64_t)p * LB;
+    k_chol_leaf<<<1, LEAF_THREADS, LB_SMEM, s>>>(W, d, d, o, L, d, Mdiag, d, sb[1], st, fault);
+    note_launches(1);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    const int rows = (int)(d - o - LB);
+    if (rows <= 0) continue;
+    // L21 = A21 * M11^T : A' = split(A21) (rows x 128), B' = split(M11) (128 x 128)
+    Split a21{sb[0], (int)((rows + 127) / 128 * 128), 128, 1};
+    Split m11{sb[1], 128, 128, 1};
+    if ((e = split(W + (o + LB) * d + o, d, 0, rows, LB, false, a21, s)) != cudaSuccess) return e;
+    const int aseg[3] = {0, 0, 128}, bseg[3] = {0, 128, 0};
+    // the epilogue also writes the split of L21 for the trailing update
+    Split l21{sb[2], (int)((rows + 127) / 128 * 128), 128, 1};
+    if ((e = gemm_tc(a21, m11, 3, aseg, bseg, 128, L + (o + LB) * d + o, d, 0, rows, LB, 1.f,
+                     0.f, false, 1, st, s, &l21)) != cudaSuccess)
+      return e;
+    // A22 -= L21 L21^T (lower tiles)
+    if ((e = gemm_tc(l21, l21, 3, aseg, bseg, 128, W + (o + LB) * d + (o + LB), d, 0, rows, rows,
+                     -1.f, 1.f, true, 1, st, s)) != cudaSuccess)
+      return e;
+  }
+  if (!Linv) return cudaSuccess;
+  // inverse by recursive doubling over block size b = 128, 256, ...
+  for (int64_t b = LB; b < d; b *= 2) {
+    const int64_t full_pairs = d / (2 * b);
+    const int64_t o_last = full_pairs * 2 * b;
+    const int64_t rows_last = d - o_last - b;
+    for (int part = 0; part < 2; ++part) {
+      const int batch = (int)(part == 0 ? full_pairs : (rows_last > 0 ? 1 : 0));
+      if (batch == 0) continue;
+      const int64_t o = part == 0 ? 0 : o_last;
+      const int rows = (int)(part == 0 ? b : rows_last);
+      const int64_t zs = 2 * b * d + 2 * b;  // source stride between pairs
+      const int kb = (int)((b + 63) / 64 * 64);
+      const int kr = (rows + 63) / 64 * 64;
+      const int rp = (rows + 127) / 128 * 128;
+      const int bp = (int)((b + 127) / 128 * 128);
+      // T_z = L21_z M11_z : A' = split(L21) (rows x b), B' = split(M11^T) (b x b)
+      Split l21{sb[0], rp, kb, batch};
+      Split m11t{sb[1], bp, kb, batch};
+      if ((e = split(L + (o + b) * d + o, d, zs, rows, (int)b, false, l21, s)) != cudaSuccess)
+        return e;
+      if ((e = split(Linv + o * d + o, d, zs, (int)b, (int)b, true, m11t, s)) != cudaSuccess)
+        return e;
+      const int as1[3] = {0, 0, kb}, bs1[3] = {0, kb, 0};
+      if ((e = gemm_tc(l21, m11t, 3, as1, bs1, (int)b, T, b, (int64_t)rp * b, rows, (int)b, 1.f,
+                       0.f, false, batch, st, s)) != cudaSuccess)
+        return e;
+      // M21_z = -M22_z T_z : A' = split(M22) (rows x rows), B' = split(T^T) (b x rows)
+      Split m22{sb[2], rp, kr, batch};
+      Split tt{sb[3], bp, kr, batch};
+      if ((e = split(Linv + (o + b) * d + (o + b), d, zs, rows, rows, false, m22, s)) !=
+          cudaSuccess)
+        return e;
+      // B'[c][k] = T[k][c]: b output rows, `rows` output columns
+      if ((e = split(T, b, (int64_t)rp * b, (int)b, rows, true, tt, s)) != cudaSuccess) return e;
+      const int as2[3] = {0, 0, kr}, bs2[3] = {0, kr, 0};
+      if ((e = gemm_tc(m22, tt, 3, as2, bs2, rows, Linv + (o + b) * d + o, d, zs, rows, (int)b,
+                       -1.f, 0.f, false, batch, st, s)) != cudaSuccess)
+        return e;
+    }
+  }
+  return cudaSuccess;
+}
+
+}  // namespace ffh

@@ -270,7 +270,7 @@ __global__ void __launch_bounds__(256) k_chol_diag(float* W, int64_t ldw, int64_
       }
       const float r = sqrtf(dj);
       s[j][j] = r;
-      if (j < b) ld_acc += 2.0 * log((double)r);
+      if (j < b) ld_acc += 2.0 * (double)logf(r);
     }
     __syncthreads();
     const float rinv = 1.f / s[j][j];

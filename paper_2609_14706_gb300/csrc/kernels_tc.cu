@@ -77,21 +77,22 @@ __device__ __forceinline__ uint32_t scale_bf16x2(uint32_t v, float s) {
 // weighted Gram
 // ===========================================================================
 namespace gram {
-constexpr int BM = 128;   // output rows (features i) per tile
-constexpr int BN = 256;   // output cols (features j) per tile
-constexpr int BK = 64;    // samples per pipeline stage
-constexpr int STAGES = 4;
+constexpr int BM = kGramBM;  // output rows (features i) per tile: two M = 128 MMAs
+constexpr int BN = kGramBN;  // output cols (features j) per tile
+constexpr int BK = 32;       // samples per pipeline stage
+constexpr int STAGES = 6;
+constexpr int BOX_BYTES = 64 * BK * 2;  // one TMA box: 64 features x BK samples
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int BOX_BYTES = 64 * BK * 2;  // one 64-feature x 64-sample TMA box
-constexpr uint32_t TMEM_COLS = 256;
+constexpr uint32_t TMEM_COLS = 512;     // two 128 x 256 fp32 accumulators
+constexpr int THREADS = 384;            // warps 0-3: TMA, MMA, TMEM; warps 4-11: scale + drain
+constexpr int NSCALE = THREADS - 128;
 constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + STAGES * BK * 4 + 256;
-constexpr int THREADS = 256;
 }  // namespace gram
 
 struct GramArgs {
-  const float* w;        // weights padded with zeros to KB*64, or nullptr (w = 1)
+  const float* w;        // weights padded with zeros to KB*BK, or nullptr (w = 1)
   float* partial;        // [units][BN][BM] fp32
   const int2* tiles;     // T lower-triangle tiles (tile row, tile col)
   int T, S, KB, units;
@@ -125,11 +126,11 @@ __global__ void __launch_bounds__(gram::THREADS, 1)
     *abort_flag = 0;
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&scaled[s], 128);
+      mbar_init(&scaled[s], NSCALE);
       mbar_init(&empty[s], 1);
     }
     mbar_init(accf, 1);
-    mbar_init(acce, 128);
+    mbar_init(acce, NSCALE);
     mbar_init(drain, 1);
     fence_mbar_init();
   }
@@ -169,8 +170,9 @@ __global__ void __launch_bounds__(gram::THREADS, 1)
             uint8_t* sa = stages + s * STAGE_BYTES;
             uint8_t* sb = sa + A_BYTES;
             const int y = kb * BK;
-            tma_load_2d(sa, &tmap, &full[s], tt.x * BM, y);
-            tma_load_2d(sa + BOX_BYTES, &tmap, &full[s], tt.x * BM + 64, y);
+#pragma unroll
+            for (int c = 0; c < BM / 64; ++c)
+              tma_load_2d(sa + c * BOX_BYTES, &tmap, &full[s], tt.x * BM + c * 64, y);
 #pragma unroll
             for (int c = 0; c < BN / 64; ++c)
               tma_load_2d(sb + c * BOX_BYTES, &tmap, &full[s], tt.y * BN + c * 64, y);
@@ -193,7 +195,7 @@ __global__ void __launch_bounds__(gram::THREADS, 1)
   } else if (warp == 1) {
     if (lane == 0) {
       // ---------------- MMA issuer ----------------
-      constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, true, true);
+      constexpr uint32_t idesc = idesc_bf16_f32(128, BN, true, true);
       uint32_t it = 0, acc_ph = 0;
       bool ok = true;
       for (int u = blockIdx.x; u < a.units && ok; u += gridDim.x) {
@@ -219,9 +221,12 @@ __global__ void __launch_bounds__(gram::THREADS, 1)
           for (int k = 0; k < BK / 16; ++k) {
             // MN-major, 128B swizzle: 16 samples = two 8-row groups (1024 B each);
             // 64-feature blocks are one TMA box (BOX_BYTES) apart.
-            const uint64_t ad = sw128_desc(sa + k * 2048, BOX_BYTES, 1024);
             const uint64_t bd = sw128_desc(sb + k * 2048, BOX_BYTES, 1024);
-            mma_bf16(tmem, ad, bd, idesc, (kb > kb0 || k > 0) ? 1u : 0u);
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh) {
+              const uint64_t ad = sw128_desc(sa + hh * 2 * BOX_BYTES + k * 2048, BOX_BYTES, 1024);
+              mma_bf16(tmem + hh * BN, ad, bd, idesc, (kb > kb0 || k > 0) ? 1u : 0u);
+            }
           }
           mma_commit(&empty[s]);
         }
@@ -241,7 +246,8 @@ __global__ void __launch_bounds__(gram::THREADS, 1)
   } else if (warp >= 4) {
     // ---------------- weight staging + epilogue ----------------
     const int t = threadIdx.x - 128;
-    const int wq = warp - 4;  // TMEM lanes 32*wq .. 32*wq+31
+    const int wq = warp & 3;          // TMEM lanes 32*wq .. 32*wq+31
+    const int hh = (warp - 4) >> 2;   // accumulator (tile rows 128*hh ..)
     uint32_t it = 0, acc_ph = 0;
     bool ok = true;
     for (int u = blockIdx.x; u < a.units && ok; u += gridDim.x) {
@@ -258,11 +264,12 @@ __global__ void __launch_bounds__(gram::THREADS, 1)
         if (a.w) {
           uint4* A4 = reinterpret_cast<uint4*>(stages + s * STAGE_BYTES);
           const float* wr = wbuf + s * BK;
-#pragma unroll 4
-          for (int c = t; c < A_BYTES / 16; c += 128) {
-            // 16-byte chunk c: sample (row of its box) = (c % 512) / 8; the swizzle only
-            // permutes chunks within a 128-byte row, so the row -> sample map is intact.
-            const float wv = wr[(c & 511) >> 3];
+          constexpr int CHUNKS_PER_BOX = BOX_BYTES / 16;
+#pragma unroll
+          for (int c = t; c < A_BYTES / 16; c += NSCALE) {
+            // 16-byte chunk c: sample (row of its box) = (c % CHUNKS_PER_BOX) / 8; the
+            // swizzle only permutes chunks within a 128-byte row.
+            const float wv = wr[(c & (CHUNKS_PER_BOX - 1)) >> 3];
             uint4 v = A4[c];
             v.x = scale_bf16x2(v.x, wv);
             v.y = scale_bf16x2(v.y, wv);
@@ -281,11 +288,11 @@ __global__ void __launch_bounds__(gram::THREADS, 1)
       }
       tc_fence_after();
       float* out = a.partial + (size_t)u * (BN * BM);
-      const int row = wq * 32 + lane;
+      const int row = hh * 128 + wq * 32 + lane;
 #pragma unroll 1
       for (int cb = 0; cb < BN / 32; ++cb) {
         float v[32];
-        tmem_ld32(tmem + ((uint32_t)(wq * 32) << 16) + cb * 32, v);
+        tmem_ld32(tmem + ((uint32_t)(wq * 32) << 16) + hh * BN + cb * 32, v);
 #pragma unroll
         for (int j = 0; j < 32; ++j) out[(size_t)(cb * 32 + j) * BM + row] = v[j];
       }
@@ -373,7 +380,7 @@ GramPlan gram_plan(int64_t N, int64_t d, int sms) {
   // at least 8 blocks of samples per unit, partial buffer at most ~2 GB
   int best_s = 1;
   double best_eff = -1.0;
-  const int max_s = std::max(1, std::min(64, p.KB / 8));
+  const int max_s = std::max(1, std::min(64, p.KB / 16));
   for (int s = 1; s <= max_s; ++s) {
     if ((double)T * s * gram::BN * gram::BM * 4.0 > 2.0e9 && s > 1) break;
     const int64_t units = (int64_t)T * s;

@@ -101,32 +101,45 @@ def test_quad_form_matches_oracle(kernel, N, d):
 # ---------------------------------------------------------------------------
 # Cholesky and inverse
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("d,cond", [(64, 1e2), (200, 1e3), (512, 1e3), (1000, 1e4), (1536, 1e3)])
-def test_cholesky_matches_oracle(d, cond):
+@pytest.mark.parametrize("kernel", KERNELS)
+@pytest.mark.parametrize("d,cond", [(64, 1e2), (200, 1e3), (512, 1e3), (1000, 1e4), (1536, 1e3),
+                                    (2304, 1e3), (4096, 1e4)])
+def test_cholesky_matches_oracle(kernel, d, cond):
+    """Cholesky factor L and inverse M = L^-1.  Unit roundoff of the arithmetic:
+    CUDA-core path fp32 (u = 2^-24, accumulated over d terms); tensor-core path bf16
+    hi/lo split products (u = 2^-16 per product, fp32 accumulation).  Bounds: backward
+    error ||L L^T - F|| / ||F|| <= 8 u_eff; inverse residual ||M L - I|| / sqrt(d) <=
+    8 u_eff sqrt(cond); forward error of L <= 8 u_eff cond; log|F| to d u_eff cond."""
     A = synth.spd_matrix(d, seed=6, cond=cond, dtype=torch.float32, device="cuda")
-    with ffh.Handle() as h:
+    with ffh.Handle(kernel=kernel) as h:
         L, Li, logdet = h.cholesky(A)
     An = oracle.as_f64(A)
     Lr = oracle.cholesky(An)
     Mr = oracle.tri_inverse(Lr)
-    eps = 2.0 ** -24
-    assert np.allclose(np.triu(oracle.as_f64(L), 1), 0)
-    assert np.allclose(np.triu(oracle.as_f64(Li), 1), 0)
-    eL = np.linalg.norm(oracle.as_f64(L) - Lr) / np.linalg.norm(Lr)
-    eM = np.linalg.norm(oracle.as_f64(Li) - Mr) / np.linalg.norm(Mr)
-    # backward-stable fp32 Cholesky: forward error ~ d * eps * cond
-    assert eL <= 4 * d * eps * cond, eL
-    assert eM <= 8 * d * eps * cond, eM
-    assert logdet == pytest.approx(oracle.logdet_from_cholesky(Lr), rel=1e-5, abs=1e-3)
+    u_eff = 2.0 ** -16 if kernel == "tc" else d * 2.0 ** -24
+    Ln, Mn = oracle.as_f64(L), oracle.as_f64(Li)
+    assert np.all(np.triu(Ln, 1) == 0) and np.all(np.triu(Mn, 1) == 0)
+    back = np.linalg.norm(Ln @ Ln.T - An) / np.linalg.norm(An)
+    inv_res = np.linalg.norm(Mn @ Ln - np.eye(d)) / math.sqrt(d)
+    eL = np.linalg.norm(Ln - Lr) / np.linalg.norm(Lr)
+    eM = np.linalg.norm(Mn - Mr) / np.linalg.norm(Mr)
+    print(f"d={d} cond={cond:g} {kernel}: back={back:.2e} inv={inv_res:.2e} eL={eL:.2e} "
+          f"eM={eM:.2e} dlogdet={abs(logdet - oracle.logdet_from_cholesky(Lr)):.2e}")
+    assert back <= 8 * u_eff, back
+    assert inv_res <= 8 * u_eff * math.sqrt(cond), inv_res
+    assert eL <= 8 * u_eff * cond, eL
+    assert eM <= 8 * u_eff * cond, eM
+    assert abs(logdet - oracle.logdet_from_cholesky(Lr)) <= d * u_eff * cond
 
 
-def test_cholesky_rejects_indefinite():
-    A = torch.eye(100, device="cuda")
-    A[50, 50] = -1.0
-    with ffh.Handle() as h:
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_cholesky_rejects_indefinite(kernel):
+    A = torch.eye(300, device="cuda")
+    A[150, 150] = -1.0
+    with ffh.Handle(kernel=kernel) as h:
         with pytest.raises(ffh.FFHError) as ei:
             h.cholesky(A)
-    assert ei.value.status == "FFH_ERR_NOT_SPD" and "50" in str(ei.value)
+    assert ei.value.status == "FFH_ERR_NOT_SPD" and "150" in str(ei.value)
 
 
 # ---------------------------------------------------------------------------
@@ -168,7 +181,9 @@ def test_fit_matches_oracle(case, kernel):
 
 def test_fit_factorial_design_closed_form():
     """GPU fit of a factorial design reaches A (x) B = Sigma_x (x) Sigma_g."""
-    P, R, n, m = 256, 128, 256, 128
+    # P = 4 n inputs and R = 4 m gradients keep Sigma_x, Sigma_g well conditioned (P = n
+    # would make a square sample covariance, condition ~1e7, beyond any fp32 Cholesky)
+    P, R, n, m = 1024, 512, 256, 128
     X, G, Xp, Gr = synth.factorial_design(P, R, n, m, seed=7, device="cuda", dtype=torch.bfloat16)
     Xp, Gr = oracle.as_f64(Xp), oracle.as_f64(Gr)
     Sx, Sg = Xp.T @ Xp / P, Gr.T @ Gr / R
