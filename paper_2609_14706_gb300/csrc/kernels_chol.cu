@@ -332,16 +332,19 @@ static cudaError_t split(const float* src, int64_t lds, int64_t src_stride, int 
 }
 
 // ---------------------------------------------------------------------------
-// 128 x 128 diagonal block: Cholesky factor L11 and inverse M11 = L11^-1 in shared
-// memory, one CTA of 512 threads.
-//   Factorisation: four 32-column sub-panels.  Within a sub-panel, each pivot step j
-//   updates only the sub-panel's columns (j, c0+32) of the rows below (one column per
-//   lane, rows spread over the 16 warps); the scaling of column j by 1/sqrt(pivot) is
-//   deferred to step j+1, which neither reads nor writes column j, so each step costs
-//   one barrier.  The finished sub-panel then updates the trailing lower triangle as a
-//   rank-32 product (4 x 4 register blocks).
-//   Inverse: the four 32 x 32 diagonal blocks by forward substitution (one warp each,
-//   lane c computes column c), then off-diagonal blocks by doubling,
+// 128 x 128 diagonal block: Cholesky factor L11 and inverse M11 = L11^-1, one CTA of
+// 512 threads (16 warps).
+//   Four 32-column sub-panels.  During a sub-panel's sweep it lives in registers:
+//   thread (warp w, lane l) holds column x = c0 + l of rows w, w+16, ..., w+112, and of
+//   the 32 x 32 diagonal block of the inverse the rows c0+w, c0+w+16.  Pivot j needs
+//   only column j of L and row j of M from other threads: their owners publish them to a
+//   double-buffered shared array at the end of pivot j-1 (one barrier per pivot).  At
+//   pivot j, x > j: L[i][x] -= l_ij l_xj (rows i > j); x <= j: M[i][x] -= l_ij m_jx
+//   (rows j < i < c0+32), the elimination applied to the identity (forward
+//   substitution in right-looking order); the owners of column j and row j scale them
+//   by 1/sqrt(pivot).  The finished sub-panel updates the trailing lower triangle as a
+//   rank-32 product in shared memory (4 x 4 register blocks).  The 128 x 128 inverse is
+//   assembled from the four 32 x 32 blocks by doubling,
 //   [[L11,0],[L21,L22]]^-1 = [[M11,0],[-M22 (L21 M11), M22]].
 // Outputs: L11 and M11 (fp32) and the bf16 hi/lo split of M11 ([hi | lo] rows, pitch
 // 256), the B operand of the panel GEMM.
@@ -380,6 +383,106 @@ __device__ __forceinline__ void smem_gemm(float* C, int ldc, const float* A, int
         *cp = accumulate ? fmaf(sgn, acc[i][j], *cp) : sgn * acc[i][j];
       }
   }
+}
+
+
+// One sub-panel sweep (Q = sub-panel index) with the panel in registers.
+// cbuf: [2][16][8] pivot-column buffer (warp-major), rbuf: [2][32] M-row buffer.
+template <int Q>
+__device__ __forceinline__ void leaf_sweep(float* Ls, float* Ms, float* cbuf, float* rbuf,
+                                           int64_t o, DevStatus* st, bool& bad) {
+  constexpr int c0 = 32 * Q;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int x = c0 + lane;
+  float a[8], m[2];
+#pragma unroll
+  for (int rr = 0; rr < 8; ++rr) {
+    const int i = warp + 16 * rr;
+    a[rr] = (i >= c0 && x <= i) ? Ls[i * LP + x] : 0.f;
+  }
+#pragma unroll
+  for (int rr = 0; rr < 2; ++rr) m[rr] = (c0 + warp + 16 * rr == x) ? 1.f : 0.f;
+  // publish column c0 (lane 0 of each warp) and row c0 of M (warp 0)
+  if (lane == 0) {
+#pragma unroll
+    for (int rr = 0; rr < 8; ++rr) cbuf[warp * 8 + rr] = a[rr];
+  }
+  if (warp == 0) rbuf[lane] = m[0];
+  __syncthreads();
+#pragma unroll 1
+  for (int jj = 0; jj < 32; ++jj) {
+    const int j = c0 + jj;
+    const float* cb = cbuf + (jj & 1) * 128;
+    const float* rb = rbuf + (jj & 1) * 32;
+    float* cbn = cbuf + ((jj + 1) & 1) * 128;
+    float* rbn = rbuf + ((jj + 1) & 1) * 32;
+    float ajj = cb[(j & 15) * 8 + (j >> 4)];
+    if (!(ajj > 0.f) || !isfinite(ajj)) {
+      if (tid == 0 && !bad) raise_error(st, FFH_ERR_NOT_SPD, (int)(o + j));
+      bad = true;
+      ajj = 1.f;
+    }
+    // 1/sqrt to within 2 ulp; far below the fp32 accumulation error of the update
+    const float rinv = rsqrtf(ajj);
+    const float r = ajj * rinv;
+    const float4 c_lo = *reinterpret_cast<const float4*>(cb + warp * 8);
+    const float4 c_hi = *reinterpret_cast<const float4*>(cb + warp * 8 + 4);
+    const float cv[8] = {c_lo.x, c_lo.y, c_lo.z, c_lo.w, c_hi.x, c_hi.y, c_hi.z, c_hi.w};
+    if (x > j) {
+      const float lxj = cb[(x & 15) * 8 + (x >> 4)] * rinv;
+#pragma unroll
+      for (int rr = 0; rr < 8; ++rr) {
+        const int i = warp + 16 * rr;
+        if (i > j && x <= i) a[rr] = fmaf(-cv[rr] * rinv, lxj, a[rr]);
+      }
+    } else {
+      const float mjx = rb[lane] * rinv;
+#pragma unroll
+      for (int rr = 0; rr < 2; ++rr) {
+        const int i = c0 + warp + 16 * rr;
+        if (i > j) m[rr] = fmaf(-cv[2 * Q + rr] * rinv, mjx, m[rr]);
+      }
+    }
+    // the owner of column j scales it (pivot -> r)
+    if (x == j) {
+#pragma unroll
+      for (int rr = 0; rr < 8; ++rr) {
+        const int i = warp + 16 * rr;
+        if (i == j)
+          a[rr] = r;
+        else if (i > j)
+          a[rr] *= rinv;
+      }
+    }
+    // the owner of row j of M scales it
+    if ((j & 15) == warp && x <= j) {
+      if (jj < 16)
+        m[0] *= rinv;
+      else
+        m[1] *= rinv;
+    }
+    // publish column j+1 of L and row j+1 of M for the next pivot
+    if (jj + 1 < 32) {
+      if (x == j + 1) {
+        *reinterpret_cast<float4*>(cbn + warp * 8) = make_float4(a[0], a[1], a[2], a[3]);
+        *reinterpret_cast<float4*>(cbn + warp * 8 + 4) = make_float4(a[4], a[5], a[6], a[7]);
+      }
+      if (((j + 1) & 15) == warp) rbn[lane] = (jj + 1 < 16) ? m[0] : m[1];
+    }
+    __syncthreads();
+  }
+  // write the finished sub-panel and the diagonal block of the inverse back
+#pragma unroll
+  for (int rr = 0; rr < 8; ++rr) {
+    const int i = warp + 16 * rr;
+    if (i >= c0 && x <= i) Ls[i * LP + x] = a[rr];
+  }
+#pragma unroll
+  for (int rr = 0; rr < 2; ++rr) {
+    const int i = c0 + warp + 16 * rr;
+    Ms[i * LP + x] = (x <= i) ? m[rr] : 0.f;
+  }
+  __syncthreads();
 }
 
 __global__ void __launch_bounds__(LEAF_THREADS) k_chol_leaf(float* W, int64_t ldw, int64_t d,
@@ -422,39 +525,15 @@ __global__ void __launch_bounds__(LEAF_THREADS) k_chol_leaf(float* W, int64_t ld
   __syncthreads();
   float ld_acc = 0.f;
   bool bad = false;
+  float* cbuf = Ts;        // [2][16][8]  (Ts is free until the doubling)
+  float* rbuf = Ts + 256;  // [2][32]
+#pragma unroll 1
   for (int q = 0; q < LB / 32; ++q) {
     const int c0 = 32 * q;
-    const int x = c0 + lane;  // this lane's column of the sub-panel
-    float rinv_prev = 1.f, r_prev = 1.f;
-    for (int jj = 0; jj <= 32; ++jj) {
-      const int j = c0 + jj;
-      // deferred scaling of column j-1 (rows >= j) and its pivot
-      if (jj > 0) {
-        if (tid < LB - j)
-          Ls[(j + tid) * LP + j - 1] *= rinv_prev;
-        else if (tid == LB - j)
-          Ls[(j - 1) * LP + j - 1] = r_prev;
-      }
-      if (jj == 32) break;
-      float ajj = Ls[j * LP + j];
-      if (!(ajj > 0.f) || !isfinite(ajj)) {
-        if (tid == 0 && !bad) raise_error(st, FFH_ERR_NOT_SPD, (int)(o + j));
-        bad = true;
-        ajj = 1.f;
-      }
-      const float r = sqrtf(ajj);
-      const float rinv = 1.f / r;
-      if (tid == 0 && j < b) ld_acc += logf(r);
-      if (x > j) {
-        const float lxj = Ls[x * LP + j] * rinv;
-        for (int i = j + 1 + ((warp - (j + 1)) & 15); i < LB; i += 16)
-          if (x <= i) Ls[i * LP + x] = fmaf(-Ls[i * LP + j] * rinv, lxj, Ls[i * LP + x]);
-      }
-      rinv_prev = rinv;
-      r_prev = r;
-      __syncthreads();
-    }
-    __syncthreads();
+    if (q == 0) leaf_sweep<0>(Ls, Ms, cbuf, rbuf, o, st, bad);
+    if (q == 1) leaf_sweep<1>(Ls, Ms, cbuf, rbuf, o, st, bad);
+    if (q == 2) leaf_sweep<2>(Ls, Ms, cbuf, rbuf, o, st, bad);
+    if (q == 3) leaf_sweep<3>(Ls, Ms, cbuf, rbuf, o, st, bad);
     // trailing rank-32 update of the lower triangle: A[r][c] -= sum_k L[r][c0+k] L[c][c0+k]
     const int r0 = c0 + 32;
     const int nb = (LB - r0) / 4;  // 4 x 4 blocks per side
@@ -483,18 +562,16 @@ __global__ void __launch_bounds__(LEAF_THREADS) k_chol_leaf(float* W, int64_t ld
     }
     __syncthreads();
   }
-  // inverse of the four 32 x 32 diagonal blocks: warp q, lane c computes column c
+  // log|F| of this block = 2 sum_i log L_ii
   if (warp < 4) {
-    const int c0 = 32 * warp, c = lane;
-    for (int i = 0; i < 32; ++i) {
-      float acc = (i == c) ? 1.f : 0.f;
-      if (i >= c) {
-        for (int k = c; k < i; ++k)
-          acc = fmaf(-Ls[(c0 + i) * LP + c0 + k], Ms[(c0 + k) * LP + c0 + c], acc);
-        Ms[(c0 + i) * LP + c0 + c] = acc / Ls[(c0 + i) * LP + c0 + i];
-      }
-    }
+    const int i = tid;
+    float lg = (i < b) ? logf(Ls[i * LP + i]) : 0.f;
+    for (int off = 16; off > 0; off >>= 1) lg += __shfl_down_sync(0xffffffffu, lg, off);
+    if (lane == 0) Ts[64 * 65 - 4 + warp] = lg;
   }
+  __syncthreads();
+  if (tid == 0)
+    ld_acc = Ts[64 * 65 - 4] + Ts[64 * 65 - 3] + Ts[64 * 65 - 2] + Ts[64 * 65 - 1];
   __syncthreads();
   // doubling, h = 32: pairs (0,1) and (2,3); h = 64: pair (0,1)
   {
