@@ -537,15 +537,213 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
 extern "C" ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_t n, int64_t m,
                                      int32_t iters, float tol, float* A_out, float* B_out) {
   if (!h) return FFH_ERR_INVALID_ARG;
-  (void)Gk;
-  (void)N;
-  (void)n;
-  (void)m;
-  (void)iters;
-  (void)tol;
-  (void)A_out;
-  (void)B_out;
-  return fail(h, FFH_ERR_UNSUPPORTED, "matrix-sample fit is not in this build");
+  h->err.clear();
+  ffh_status vs = validate_opt(h);
+  if (vs) return vs;
+  if (!Gk || !A_out || !B_out) return fail(h, FFH_ERR_INVALID_ARG, "null pointer argument");
+  if (N < 1 || n < 1 || m < 1 || iters < 1)
+    return fail(h, FFH_ERR_INVALID_ARG, "need N, n, m, iters >= 1");
+  if (n % 8 || m % 8) return fail(h, FFH_ERR_INVALID_ARG, "matrix samples need n, m multiples of 8");
+  if (!(tol >= 0.f) || !std::isfinite(tol)) return fail(h, FFH_ERR_INVALID_ARG, "tol must be finite and >= 0");
+  if (h->opt.kernel != 0) return fail(h, FFH_ERR_UNSUPPORTED, "matrix samples need the tensor-core kernels");
+  if (h->opt.variant != FFH_FLIPFLOP) return fail(h, FFH_ERR_UNSUPPORTED, "matrix samples: FlipFlop variant only");
+  if (N * std::min(n, m) < std::max(n, m) && h->opt.damping == 0.f)
+    return fail(h, FFH_ERR_RANK, "N min(n, m) < max(n, m) without damping");
+  if (N * m > ((int64_t)1 << 31) - 1 || N * n > ((int64_t)1 << 31) - 1)
+    return fail(h, FFH_ERR_INVALID_ARG, "N * max(n, m) too large");
+  const bool g_dev = is_device_ptr(Gk);
+  const bool init = h->opt.init_A != nullptr;
+  const int64_t D = std::max(n, m);
+  const int64_t mn = m * n;
+  // samples per chunk: transform output (V) chunk of about 1 GiB
+  const int64_t Kc = std::max<int64_t>(1, std::min<int64_t>(N, ((int64_t)1 << 29) / mn));
+  const int64_t Kh = g_dev ? 0 : Kc;  // host staging (fp32) chunk
+  GramPlan pa = gram_plan(Kc * m, n, num_sms()), pb = gram_plan(Kc * n, m, num_sms());
+  const int nt = (int)((D + 63) / 64);
+  auto layout = [&](Carve& c, DevStatus** st, IterRecord** recs, __nv_bfloat16** Gb,
+                    float** stage, __nv_bfloat16** V, float** A2, float** B2, float** Cc,
+                    float** L, float** Linv, __nv_bfloat16** Mb, float** work, float** DI,
+                    int2** tn, int** ln, int2** tm, int** lm, float** partial, double** trb,
+                    double** fro) {
+    *st = c.take<DevStatus>(1);
+    *recs = c.take<IterRecord>(iters + 2);
+    *Gb = c.take<__nv_bfloat16>((size_t)N * mn);
+    *stage = Kh ? c.take<float>((size_t)Kh * mn) : nullptr;
+    *V = c.take<__nv_bfloat16>((size_t)Kc * mn);
+    *A2 = c.take<float>((size_t)2 * n * n);
+    *B2 = c.take<float>((size_t)2 * m * m);
+    *Cc = c.take<float>((size_t)D * D);
+    *L = c.take<float>((size_t)D * D);
+    *Linv = c.take<float>((size_t)D * D);
+    *Mb = c.take<__nv_bfloat16>((size_t)D * D);
+    *work = c.take<float>(std::max(cholesky_work_floats(D), cholesky_tc_work_bytes(D) / 4 + 1));
+    *DI = c.take<float>((size_t)nt * 64 * 64);
+    *tn = c.take<int2>(gram_tile_table_bytes(n) / sizeof(int2) + 1);
+    *ln = c.take<int>(gram_tile_table_bytes(n) / sizeof(int) + 1);
+    *tm = c.take<int2>(gram_tile_table_bytes(m) / sizeof(int2) + 1);
+    *lm = c.take<int>(gram_tile_table_bytes(m) / sizeof(int) + 1);
+    *partial = c.take<float>(std::max(gram_partial_bytes(pa), gram_partial_bytes(pb)) / 4);
+    *trb = c.take<double>(8);
+    *fro = c.take<double>(4);
+  };
+  DevStatus* st;
+  IterRecord* recs;
+  __nv_bfloat16 *Gb, *V, *Mb;
+  float *stage, *A2, *B2, *Cc, *L, *Linv, *work, *DI, *partial;
+  int2 *tn, *tm;
+  int *ln, *lm;
+  double *trb, *fro;
+  {
+    Carve c(nullptr);
+    layout(c, &st, &recs, &Gb, &stage, &V, &A2, &B2, &Cc, &L, &Linv, &Mb, &work, &DI, &tn, &ln,
+           &tm, &lm, &partial, &trb, &fro);
+    ffh_status es = ensure_ws(h, c.off + 1024);
+    if (es) return es;
+  }
+  Carve c(h->ws);
+  layout(c, &st, &recs, &Gb, &stage, &V, &A2, &B2, &Cc, &L, &Linv, &Mb, &work, &DI, &tn, &ln, &tm,
+         &lm, &partial, &trb, &fro);
+  cudaStream_t s = h->stream;
+  CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
+  CK(cudaMemsetAsync(recs, 0, sizeof(IterRecord) * (iters + 2), s));
+  GramTables gtn, gtm;
+  {
+    // the Gram plans depend on the chunk length; tables depend on d only
+    ffh_status es = setup_tables(h, Kc * m, n, &gtn, tn, ln);
+    if (es) return es;
+    es = setup_tables(h, Kc * n, m, &gtm, tm, lm);
+    if (es) return es;
+  }
+  // samples -> bf16 (N*m rows of n)
+  for (int64_t k0 = 0; k0 < N; k0 += (g_dev ? N : Kh)) {
+    const int64_t nk = std::min(N - k0, g_dev ? N : Kh);
+    const float* src = Gk + k0 * mn;
+    if (!g_dev) {
+      CK(cudaMemcpyAsync(stage, src, sizeof(float) * nk * mn, cudaMemcpyHostToDevice, s));
+      src = stage;
+    }
+    CK(launch_to_bf16(src, nk * m, n, n, Gb + k0 * mn, n, s));
+  }
+  float* A[2] = {A2, A2 + (size_t)n * n};
+  float* B[2] = {B2, B2 + (size_t)m * m};
+  int cur = 0;
+  if (init) {
+    CK(cudaMemcpyAsync(A[cur], h->opt.init_A, sizeof(float) * n * n, cudaMemcpyDefault, s));
+  } else {
+    CK(launch_fill_identity(A[cur], n, n, s));
+  }
+  const float lam = h->opt.damping;
+  const float sB = (float)(1.0 / ((double)N * (double)n));
+  const float sA = (float)(1.0 / ((double)N * (double)m));
+  ffh_status es;
+  // one half-step: C = scale * sum over chunks of Gram(M * Gop_k)
+  auto half = [&](const __nv_bfloat16* Mbf, int64_t d, bool b_update, float scale, float* C,
+                  const GramTables& gt) -> ffh_status {
+    const int64_t d_other = b_update ? m : n;
+    CK(cudaMemsetAsync(C, 0, sizeof(float) * d_other * d_other, s));
+    for (int64_t k0 = 0; k0 < N; k0 += Kc) {
+      const int64_t nk = std::min(Kc, N - k0);
+      CK(launch_transform_tc(Mbf, d, d, Gb + k0 * mn, nk, m, n, b_update, V, st, s));
+      Staged vsd;
+      vsd.bf = V;
+      vsd.ld_bf = d_other;
+      vsd.raw = V;
+      vsd.ld_raw = d_other;
+      GramTables g2 = gt;
+      g2.plan = gram_plan(nk * d, d_other, num_sms());
+      // the partial buffer holds the split count of a full chunk; never exceed it
+      const GramPlan& full = b_update ? pb : pa;
+      if (g2.plan.units > full.units) {
+        g2.plan.S = std::max(1, full.units / g2.plan.T);
+        g2.plan.units = g2.plan.T * g2.plan.S;
+        g2.plan.grid = std::min(g2.plan.units, num_sms());
+      }
+      ffh_status e2 = gram(h, vsd, nk * d, d_other, nullptr, scale, Cc, partial, g2, st);
+      if (e2) return e2;
+      CK(launch_add(C, Cc, d_other * d_other, s));
+    }
+    return FFH_OK;
+  };
+  int t_done = 0;
+  std::vector<IterRecord> host_recs((size_t)iters + 2);
+  for (int t = 1; t <= iters; ++t) {
+    IterRecord* R = recs + t;
+    const int nxt = cur ^ 1;
+    // ---- M_A = chol(A_{t-1})^-1 (bf16)
+    es = chol(h, A[cur], n, L, Linv, work, DI, st, 0);
+    if (es) return es;
+    CK(cudaMemcpyAsync(&R->logdet_A_prev, &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
+    if (t > 1) {
+      CK(cudaMemcpyAsync(&recs[t - 1].logdet_A, &st->logdet, sizeof(double),
+                         cudaMemcpyDeviceToDevice, s));
+      CK(launch_frob2(Linv, n, &recs[t - 1].trinvA, s));
+    }
+    CK(launch_lower_to_bf16(Linv, n, n, Mb, n, s));
+    // ---- B-update
+    es = half(Mb, n, true, sB, B[nxt], gtm);
+    if (es) return es;
+    CK(launch_damp(B[nxt], m, m, lam, st, s, &R->shift_B));
+    es = chol(h, B[nxt], m, L, Linv, work, DI, st,
+              (t == 1 && h->opt.fault == FFH_FAULT_BAD_PIVOT) ? FFH_FAULT_BAD_PIVOT : 0);
+    if (es) return es;
+    CK(cudaMemcpyAsync(&R->logdet_B, &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
+    CK(launch_frob2(Linv, m, &R->trinvB, s));
+    CK(launch_lower_to_bf16(Linv, m, m, Mb, m, s));
+    // ---- A-update
+    es = half(Mb, m, false, sA, A[nxt], gtn);
+    if (es) return es;
+    CK(launch_damp(A[nxt], n, n, lam, st, s, &R->shift_A));
+    CK(launch_normalize(A[nxt], n, B[nxt], m, R, st, s));
+    CK(cudaMemsetAsync(&R->dA2, 0, sizeof(double) * 4, s));
+    CK(launch_trace(A[nxt], n, trb + 0, s));
+    CK(launch_trace(A[cur], n, trb + 1, s));
+    CK(launch_delta(A[nxt], A[cur], n, &R->dA2, &R->nA2, trb, s));
+    if (t > 1) {
+      CK(launch_trace(B[nxt], m, trb + 2, s));
+      CK(launch_trace(B[cur], m, trb + 3, s));
+      CK(launch_delta(B[nxt], B[cur], m, &R->dB2, &R->nB2, trb + 2, s));
+    }
+    cur = nxt;
+    t_done = t;
+    if (tol > 0.f && t > 1) {
+      IterRecord hr;
+      CK(cudaMemcpyAsync(&hr, R, sizeof(hr), cudaMemcpyDeviceToHost, s));
+      CK(cudaStreamSynchronize(s));
+      const double dA = hr.nA2 > 0 ? std::sqrt(hr.dA2 / hr.nA2) : 0.0;
+      const double dB = hr.nB2 > 0 ? std::sqrt(hr.dB2 / hr.nB2) : 0.0;
+      if (std::max(dA, dB) < (double)tol) break;
+    }
+  }
+  if (h->opt.final_loglik) {
+    es = chol(h, A[cur], n, L, Linv, work, DI, st, 0);
+    if (es) return es;
+    CK(cudaMemcpyAsync(&recs[t_done].logdet_A, &st->logdet, sizeof(double),
+                       cudaMemcpyDeviceToDevice, s));
+    CK(launch_frob2(Linv, n, &recs[t_done].trinvA, s));
+  }
+  CK(cudaMemcpyAsync(A_out, A[cur], sizeof(float) * n * n, cudaMemcpyDefault, s));
+  CK(cudaMemcpyAsync(B_out, B[cur], sizeof(float) * m * m, cudaMemcpyDefault, s));
+  CK(cudaMemcpyAsync(host_recs.data(), recs, sizeof(IterRecord) * (iters + 2),
+                     cudaMemcpyDeviceToHost, s));
+  es = read_status(h, st);
+  // trace terms of the log-likelihood from exact identities:
+  //   sum_k tr(B^-1 G_k A^-1 G_k^T) = N n tr(B^-1 S_B) = N n (m - shift_B tr(B^-1)) at the
+  //   B-point (B = S_B + shift_B I), and N m (n - shift_A tr(A^-1)) at the A-point.
+  const double Nd = (double)N, nd = (double)n, md = (double)m;
+  for (int t = 1; t <= t_done; ++t) {
+    IterRecord& R = host_recs[t];
+    R.sum_qr_B = Nd * nd * (md - R.shift_B * R.trinvB);
+    const bool haveA = t < t_done || h->opt.final_loglik;
+    // trinvA is of the rescaled A_t; the shift is in the units before the rescale
+    R.sum_qr_A = haveA ? R.scale * Nd * md * (nd - R.shift_A * R.trinvA / R.scale) : 0.0;
+  }
+  h->iters_done = t_done;
+  h->N = N;
+  h->n = n;
+  h->m = m;
+  h->final_loglik = h->opt.final_loglik != 0;
+  h->recs = host_recs;
+  return es;
 }
 
 extern "C" ffh_status ffh_get_stats(ffh_t h, int32_t* iters_done, double* delta,

@@ -33,7 +33,10 @@ struct IterRecord {
   double dA2, nA2;       // ||A^_t - A^_{t-1}||^2, ||A^_t||^2
   double dB2, nB2;       // same for B
   double trB;            // tr(B_t) after the rescale
-  double pad;
+  double shift_B;        // damping shift added to B_t (0 undamped)
+  double shift_A;        // damping shift added to A_t before the rescale
+  double trinvB;         // tr(B_t^-1) = ||L_B^-1||_F^2 (matrix-sample fit)
+  double trinvA;         // tr(A_t^-1) after the rescale (filled by the next iteration)
 };
 
 __device__ __forceinline__ void raise_error(DevStatus* st, int code, int info) {
@@ -103,7 +106,12 @@ cudaError_t launch_cholesky_tc(const float* F, int64_t d, int64_t ldf, float* L,
 size_t cholesky_tc_work_bytes(int64_t d);
 cudaError_t launch_fill_identity(float* F, int64_t d, int64_t ld, cudaStream_t s);
 cudaError_t launch_damp(float* F, int64_t d, int64_t ld, float lambda, DevStatus* st,
-                        cudaStream_t s);
+                        cudaStream_t s, double* shift_out = nullptr);
+cudaError_t launch_add(float* C, const float* X, int64_t total, cudaStream_t s);
+// matrix samples (kernels_matrix.cu): V rows (k, r) = (M Gop_k)[r][:], see the file
+cudaError_t launch_transform_tc(const __nv_bfloat16* M, int64_t d, int64_t ldm,
+                                const __nv_bfloat16* Gb, int64_t nk, int64_t m, int64_t n,
+                                bool b_update, __nv_bfloat16* V, DevStatus* st, cudaStream_t s);
 // A <- A / s, B <- B * s with s = tr(A)/n; records s and log-determinant corrections
 cudaError_t launch_normalize(float* A, int64_t n, float* B, int64_t m, IterRecord* rec,
                              DevStatus* st, cudaStream_t s);

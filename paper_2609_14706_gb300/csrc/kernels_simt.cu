@@ -444,8 +444,9 @@ cudaError_t launch_fill_identity(float* F, int64_t d, int64_t ld, cudaStream_t s
   return cudaGetLastError();
 }
 
-// F += lambda * mean(diag F) * I (mean taken before the shift)
-__global__ void k_damp(float* F, int64_t d, int64_t ld, float lambda) {
+// F += lambda * mean(diag F) * I (mean taken before the shift); the shift is also
+// written to *shift_out when given
+__global__ void k_damp(float* F, int64_t d, int64_t ld, float lambda, double* shift_out) {
   double acc = 0.0;
   for (int64_t i = threadIdx.x; i < d; i += blockDim.x) acc += F[i * ld + i];
   __shared__ double tot;
@@ -454,12 +455,29 @@ __global__ void k_damp(float* F, int64_t d, int64_t ld, float lambda) {
   __syncthreads();
   const float shift = (float)((double)lambda * tot / (double)d);
   for (int64_t i = threadIdx.x; i < d; i += blockDim.x) F[i * ld + i] += shift;
+  if (threadIdx.x == 0 && shift_out) *shift_out = (double)shift;
 }
 
 cudaError_t launch_damp(float* F, int64_t d, int64_t ld, float lambda, DevStatus*,
-                        cudaStream_t s) {
-  if (lambda == 0.f) return cudaSuccess;
-  k_damp<<<1, 1024, 0, s>>>(F, d, ld, lambda); note_launches(1);
+                        cudaStream_t s, double* shift_out) {
+  if (lambda == 0.f) return shift_out ? cudaMemsetAsync(shift_out, 0, sizeof(double), s)
+                                      : cudaSuccess;
+  k_damp<<<1, 1024, 0, s>>>(F, d, ld, lambda, shift_out);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+// C += X (d x d, same pitch)
+__global__ void k_add(float* C, const float* X, int64_t total) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+       i += (int64_t)gridDim.x * blockDim.x)
+    C[i] += X[i];
+}
+
+cudaError_t launch_add(float* C, const float* X, int64_t total, cudaStream_t s) {
+  const int64_t blocks = std::min<int64_t>((total + 255) / 256, (int64_t)num_sms() * 8);
+  k_add<<<(unsigned)std::max<int64_t>(1, blocks), 256, 0, s>>>(C, X, total);
+  note_launches(1);
   return cudaGetLastError();
 }
 

@@ -265,3 +265,41 @@ def test_fault_injection_oom_and_pivot():
     with ffh.Handle(dtype="bf16") as h:
         A, B = h.fit(X, G, iters=1)
     assert torch.isfinite(A).all()
+
+
+# ---------------------------------------------------------------------------
+# matrix samples (Section 5, general G_k)
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("N,n,m,iters", [(256, 64, 96, 5), (300, 136, 72, 4), (96, 512, 768, 3)])
+def test_fit_matrix_matches_oracle(N, n, m, iters):
+    wl = synth.WORKLOADS["kron_recovery_512x768"].with_(n=n, m=m)
+    Gk = synth.matrix_samples(wl, seed=3, device="cuda", N=N)
+    with ffh.Handle(dtype="f32", final_loglik=True) as h:
+        A, B = h.fit_matrix(Gk, iters=iters)
+        st = h.stats()
+    ref = oracle.flipflop_fit_matrix(Gk.cpu(), iters=iters)
+    err = oracle.kron_rel_err(A.cpu(), B.cpu(), ref.A, ref.B)
+    assert err <= 2e-3, err
+    assert st["iters_done"] == iters
+    assert np.allclose(st["mean_qr"], m * n, rtol=1e-6)
+    assert np.allclose(st["loglik"], ref.loglik, rtol=1e-3, atol=1e-3 * np.abs(ref.loglik).max())
+
+
+def test_fit_matrix_rank_one_samples_equal_rank_one_fit():
+    """G_k = g_k x_k^T: the matrix-sample fit and the rank-one fit agree."""
+    wl = synth.WORKLOADS["llama7b_attn_4096"].with_(N=2048, n=128, m=64, iters=3, dtype="f32")
+    X, G = synth.rank_one_samples(wl, seed=0, device="cuda")
+    Gk = torch.einsum("ki,kj->kij", G, X).contiguous()
+    with ffh.Handle(dtype="f32") as h:
+        A1, B1 = h.fit(X, G, iters=3)
+        A2, B2 = h.fit_matrix(Gk, iters=3)
+    assert oracle.kron_rel_err(A2.cpu(), B2.cpu(), A1.cpu(), B1.cpu()) <= 2e-3
+
+
+def test_fit_matrix_host_input_and_damping():
+    wl = synth.WORKLOADS["kron_recovery_512x768"].with_(n=64, m=48)
+    Gk = synth.matrix_samples(wl, seed=4, device="cuda", N=200)
+    with ffh.Handle(dtype="f32", damping=0.1) as h:
+        A, B = h.fit_matrix(Gk.cpu(), iters=3)
+    ref = oracle.flipflop_fit_matrix(Gk.cpu(), iters=3, damping=0.1)
+    assert oracle.kron_rel_err(A, B, ref.A, ref.B) <= 2e-3
