@@ -18,9 +18,11 @@ problems, weak scaling, no collective in the data path); rank 0 prints the line.
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import math
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -59,6 +61,25 @@ def measured_peaks():
     except OSError:
         return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, \
             "fallback"
+
+
+def profiled_traffic(workload: str):
+    """DRAM bytes per launch of the Gram kernel from the committed ncu summary, if the
+    kernel source is still the one that was profiled (else None)."""
+    path = os.path.join(ROOT, "profiles", f"k_gram_tc_{workload}.md")
+    try:
+        text = open(path).read()
+    except OSError:
+        return None
+    m1 = re.search(r"source_sha256:\s*([0-9a-f]{64})", text)
+    m2 = re.search(r"traffic_bytes_per_launch:\s*(\d+)", text)
+    if not (m1 and m2):
+        return None
+    src = os.path.join(ROOT, "paper_2609_14706_gb300", "csrc", "kernels_tc.cu")
+    with open(src, "rb") as f:
+        if hashlib.sha256(f.read()).hexdigest() != m1.group(1):
+            return None
+    return int(m2.group(1))
 
 
 # ---------------------------------------------------------------------------
@@ -200,18 +221,29 @@ def run_ours(args):
         dist_mod.init_process_group("nccl")
         dist = dist_mod
     wl = synth.WORKLOADS[args.workload]
-    if wl.kind != "rank_one":
-        raise SystemExit("bench.py times the rank-one fit")
+    matrix = wl.kind == "matrix"
     iters = wl.iters
-    # each rank fits its own layer (independent problems)
-    X, G = synth.rank_one_samples(wl, seed=args.seed + rank, device="cuda")
     N, n, m = wl.N, wl.n, wl.m
+    # each rank fits its own layer (independent problems)
+    if matrix:
+        Gk = synth.matrix_samples(wl, seed=args.seed + rank, device="cuda")
+    else:
+        X, G = synth.rank_one_samples(wl, seed=args.seed + rank, device="cuda")
     A = torch.empty(n, n, dtype=torch.float32, device="cuda")
     B = torch.empty(m, m, dtype=torch.float32, device="cuda")
     stream = torch.cuda.current_stream()
     h = ffh.Handle(dtype=wl.dtype, profile=True, stream=stream)
+
+    def one_fit(hh, a_out, b_out, host=False):
+        if matrix:
+            hh.fit_matrix(Gk, iters, 0.0, a_out, b_out)
+        elif host:
+            hh.fit(Xh, Gh, iters, 0.0, a_out, b_out)
+        else:
+            hh.fit(X, G, iters, 0.0, a_out, b_out)
+
     for _ in range(max(args.warmup, 3)):
-        h.fit(X, G, iters, 0.0, A, B)
+        one_fit(h, A, B)
     torch.cuda.synchronize()
     h.timings(reset=True)
     launches0 = h.timings()["kernel_launches"]
@@ -227,7 +259,7 @@ def run_ours(args):
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for _ in range(args.steps):
-        h.fit(X, G, iters, 0.0, A, B)
+        one_fit(h, A, B)
     e1.record(stream)
     barrier()
     clk = clocks.stop()
@@ -242,20 +274,20 @@ def run_ours(args):
 
     # ---- end to end through the C ABI with host buffers
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and not matrix:
         Xh = X.cpu().pin_memory()
         Gh = G.cpu().pin_memory()
         Ah = torch.empty(n, n, dtype=torch.float32).pin_memory()
         Bh = torch.empty(m, m, dtype=torch.float32).pin_memory()
         h2 = ffh.Handle(dtype=wl.dtype, stream=stream)
-        h2.fit(Xh, Gh, iters, 0.0, Ah, Bh)
+        one_fit(h2, Ah, Bh, host=True)
         barrier()
         t0 = time.perf_counter()
         f0 = torch.cuda.Event(enable_timing=True)
         f1 = torch.cuda.Event(enable_timing=True)
         f0.record(stream)
         for _ in range(args.steps):
-            h2.fit(Xh, Gh, iters, 0.0, Ah, Bh)
+            one_fit(h2, Ah, Bh, host=True)
         f1.record(stream)
         barrier()
         wall_ms = (time.perf_counter() - t0) * 1e3
@@ -272,16 +304,22 @@ def run_ours(args):
 
     # ---- roofline of the dominant kernel (weighted Gram), measured live above
     peaks, peak_kind = measured_peaks()
-    gram_flops_step = iters * (ffh.gram_flops(N, n) + ffh.gram_flops(N, m))
+    if matrix:
+        # Grams over N m rows of n features and N n rows of m features
+        gram_flops_step = iters * (ffh.gram_flops(N * m, n) + ffh.gram_flops(N * n, m))
+    else:
+        gram_flops_step = iters * (ffh.gram_flops(N, n) + ffh.gram_flops(N, m))
     gram_tflops = (gram_flops_step * args.steps) / (tim["gram_ms"] / 1e3) / 1e12
     peak = float(peaks.get("bf16_tflops_sustained", peaks.get("bf16_tflops")))
-    qform_flops_step = iters * (ffh.qform_flops(N, n) + ffh.qform_flops(N, m))
-    qform_tflops = (qform_flops_step * args.steps) / (tim["qform_ms"] / 1e3) / 1e12
+    qform_flops_step = 0.0 if matrix else iters * (ffh.qform_flops(N, n) + ffh.qform_flops(N, m))
+    qform_tflops = ((qform_flops_step * args.steps) / (tim["qform_ms"] / 1e3) / 1e12
+                    if tim["qform_ms"] > 0 else None)
     roofline = {"bound": "tensor", "kernel": "k_gram_tc (weighted Gram)",
                 "achieved": gram_tflops, "peak": peak, "unit": "TFLOP/s",
-                "frac": gram_tflops / peak, "traffic": None,
+                "frac": gram_tflops / peak, "traffic": profiled_traffic(wl.name),
+                "traffic_unit": "bytes per launch (ncu dram__bytes_read + write)",
                 "peak_source": f"{peak_kind} bf16 dense, sustained (kernel timed inside a long step)",
-                "flops_per_launch": (ffh.gram_flops(N, n) + ffh.gram_flops(N, m)) / 2,
+                "flops_per_launch": gram_flops_step * args.steps / max(1, tim["gram_launches"]),
                 "avg_launch_ms": tim["gram_ms"] / max(1, tim["gram_launches"])}
     kernels = {
         "gram_ms_per_step": tim["gram_ms"] / args.steps,
@@ -292,7 +330,7 @@ def run_ours(args):
     }
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and not matrix:
         ns = oracle_sample_size(wl)
         t_full, t_sample = oracle_iteration_seconds(wl, X[:ns].cpu(), G[:ns].cpu(), ns)
         cpu = {"value": 1.0 / t_full, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
@@ -302,7 +340,7 @@ def run_ours(args):
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32",
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic",
         "config": {"workload": wl.name, "N": N, "n": n, "m": m, "iters_per_step": iters,
                    "parallelism": f"replicas{world}" if world > 1 else "single",
