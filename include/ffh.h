@@ -55,10 +55,15 @@ typedef enum {
 
 typedef enum { FFH_BF16 = 0, FFH_F32 = 1 } ffh_dtype;
 
-/* Hessian variants of Table 1 that share the alternating loop. */
+/* The Hessian approximations of Table 1 (all returned with tr(A) = n, B carrying the
+ * scale; only the product A (x) B is defined by the paper). */
 typedef enum {
   FFH_FLIPFLOP = 0,  /* A = E[(g^T B^-1 g) x x^T], B = E[(x^T A^-1 x) g g^T] (Section 5) */
-  FFH_FROBENIUS = 1  /* A = E[(g^T B g) x x^T]/||B||_F^2, B = E[(x^T A x) g g^T]/||A||_F^2 */
+  FFH_FROBENIUS = 1, /* A = E[(g^T B g) x x^T]/||B||_F^2, B = E[(x^T A x) g g^T]/||A||_F^2:
+                        alternating least squares for min ||H - A (x) B||_F (Section 5,
+                        last paragraph); same A_0 = I and B-then-A order */
+  FFH_INPUT = 2,     /* A = E[x x^T], B = I_m (one pass; iters ignored) */
+  FFH_MARGINAL = 3   /* A = E[x x^T], B = E[g g^T] (one pass; iters ignored) */
 } ffh_variant;
 
 /* Test-only fault injection codes (ffh_options.fault). */
@@ -158,6 +163,16 @@ ffh_status ffh_get_stats(ffh_t h, int32_t* iters_done, double* delta, double* lo
 /* Copy the accumulated timings into *out; reset = 1 clears them afterwards (the
  * process-wide launch counter is not reset). */
 ffh_status ffh_get_timings(ffh_t h, ffh_timings* out, int32_t reset);
+
+/* Scale-free mismatch factor of a Kronecker approximation (Section 4, its definition,
+ * in the sample form of Section 5):
+ *   Phi~(A, B) = |A|^{1/n} |B|^{1/m} (1/(N m n)) sum_k (x_k^T A^-1 x_k)(g_k^T B^-1 g_k)
+ * which is Phi(H, A (x) B) times |H|^{1/mn} (H need not be invertible).  Smaller is
+ * better; the FlipFlop fit minimises it.
+ *   X, G: samples as for ffh_fit (device), A (n x n), B (m x m): fp32 SPD (device)
+ *   phi_out: host double.  Errors: INVALID_ARG, NOT_SPD, CUDA. */
+ffh_status ffh_phi_tilde(ffh_t h, const void* X, const void* G, int64_t N, int64_t n, int64_t m,
+                         const float* A, const float* B, double* phi_out);
 
 /* ---- single steps of the fit (device pointers only; on the handle's stream) ---- */
 

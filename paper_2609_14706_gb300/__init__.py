@@ -26,7 +26,9 @@ HEADER_PATH = os.path.join(os.path.dirname(_HERE), "include", "ffh.h")
 STATUS = {0: "FFH_OK", 1: "FFH_ERR_INVALID_ARG", 2: "FFH_ERR_NOT_SPD", 3: "FFH_ERR_RANK",
           4: "FFH_ERR_OOM", 5: "FFH_ERR_CUDA", 6: "FFH_ERR_TIMEOUT", 7: "FFH_ERR_UNSUPPORTED"}
 FFH_BF16, FFH_F32 = 0, 1
-FFH_FLIPFLOP, FFH_FROBENIUS = 0, 1
+FFH_FLIPFLOP, FFH_FROBENIUS, FFH_INPUT, FFH_MARGINAL = 0, 1, 2, 3
+VARIANTS = {"flipflop": FFH_FLIPFLOP, "frobenius": FFH_FROBENIUS, "input": FFH_INPUT,
+            "marginal": FFH_MARGINAL}
 FAULT_NONE, FAULT_OOM, FAULT_BAD_PIVOT, FAULT_LOST_COPY = 0, 1, 2, 3
 
 
@@ -83,6 +85,7 @@ def load_library(path: Optional[str] = None):
         "ffh_get_timings": ([vp, ctypes.POINTER(ffh_timings), i32], ctypes.c_int),
         "ffh_weighted_gram_static": ([vp, vp, i64, i64, f32, vp, vp, ctypes.c_char_p, i32],
                                      ctypes.c_int),
+        "ffh_phi_tilde": ([vp, vp, vp, i64, i64, i64, vp, vp, pd], ctypes.c_int),
     }
     for name, (args, res) in sigs.items():
         fn = getattr(lib, name)
@@ -130,7 +133,7 @@ class Handle:
         self.opts = ffh_options()
         self.opts.dtype = _dtype_code(dtype)
         self.opts.damping = float(damping)
-        self.opts.variant = {"flipflop": FFH_FLIPFLOP, "frobenius": FFH_FROBENIUS}[variant]
+        self.opts.variant = VARIANTS[variant]
         if init_A is not None:
             init_A = init_A.to(torch.float32).contiguous()
             self._keep.append(init_A)
@@ -225,6 +228,20 @@ class Handle:
         code = self._lib.ffh_get_timings(self._h, ctypes.byref(t), int(bool(reset)))
         _check(self._lib, self._h, code, "ffh_get_timings")
         return {f: getattr(t, f) for f, _ in ffh_timings._fields_}
+
+    def phi_tilde(self, X: torch.Tensor, G: torch.Tensor, A: torch.Tensor,
+                  B: torch.Tensor) -> float:
+        """ffh_phi_tilde: scale-free mismatch factor of A (x) B on the samples."""
+        X, G = self._samples(X, "X"), self._samples(G, "G")
+        N, n = X.shape
+        m = G.shape[1]
+        A = A.to(torch.float32).contiguous()
+        B = B.to(torch.float32).contiguous()
+        out = ctypes.c_double()
+        code = self._lib.ffh_phi_tilde(self._h, _ptr(X), _ptr(G), N, n, m, _ptr(A), _ptr(B),
+                                       ctypes.byref(out))
+        _check(self._lib, self._h, code, "ffh_phi_tilde")
+        return out.value
 
     # -- single steps --
     def weighted_gram(self, V: torch.Tensor, w: Optional[torch.Tensor], scale: float = 1.0,

@@ -39,6 +39,7 @@ struct ffh_ctx {
   int iters_done = 0;
   int64_t N = 0, n = 0, m = 0;
   bool final_loglik = false;
+  bool loglik_valid = true;      // the FlipFlop log-likelihood applies to the last fit
   std::vector<IterRecord> recs;  // index 1..iters_done
   // profiling (opt.profile): CUDA events recorded around the timed kernels
   double prof_ms[3] = {0, 0, 0};        // gram, qform, cholesky
@@ -251,7 +252,7 @@ ffh_status validate_opt(ffh_t h) {
   if (o.dtype != FFH_BF16 && o.dtype != FFH_F32) return fail(h, FFH_ERR_INVALID_ARG, "bad dtype %d", o.dtype);
   if (!(o.damping >= 0.f) || !std::isfinite(o.damping))
     return fail(h, FFH_ERR_INVALID_ARG, "damping must be finite and >= 0");
-  if (o.variant != FFH_FLIPFLOP && o.variant != FFH_FROBENIUS)
+  if (o.variant < FFH_FLIPFLOP || o.variant > FFH_MARGINAL)
     return fail(h, FFH_ERR_INVALID_ARG, "bad variant %d", o.variant);
   if (o.kernel != 0 && o.kernel != 1) return fail(h, FFH_ERR_INVALID_ARG, "bad kernel %d", o.kernel);
   return FFH_OK;
@@ -299,6 +300,23 @@ ffh_status gram(ffh_t h, const Staged& V, int64_t N, int64_t d, const float* w_p
     CK(launch_gram_tc(V.bf, N, d, V.ld_bf, w_padded, scale, C, d, partial, gt.tiles, gt.lut,
                       gt.plan, st, h->opt.fault, h->stream, t1));
     prof_end(h, PROF_GRAM, t0, t1);
+  }
+  return FFH_OK;
+}
+
+// q_k = ||L^T v_k||^2 = v_k^T F v_k for F = L L^T (the Frobenius variant's weights)
+ffh_status qform_fwd(ffh_t h, const Staged& V, int64_t N, int64_t d, const float* L,
+                     const float* F, __nv_bfloat16* Mb, float* q, DevStatus* st) {
+  if (h->opt.kernel == 1) {
+    cudaEvent_t t0 = prof_begin(h);
+    CK(launch_fwd_qform_simt(V.raw, h->opt.dtype, N, d, V.ld_raw, F, d, q, h->stream));
+    prof_end(h, PROF_QFORM, t0);
+  } else {
+    const int64_t ldm = pad8(d);
+    CK(launch_lowerT_to_bf16(L, d, d, Mb, ldm, h->stream));
+    cudaEvent_t t0 = prof_begin(h);
+    CK(launch_qform_tc(V.bf, N, d, V.ld_bf, Mb, ldm, q, st, h->stream, true));
+    prof_end(h, PROF_QFORM, t0);
   }
   return FFH_OK;
 }
@@ -363,8 +381,6 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
   if (!(tol >= 0.f) || !std::isfinite(tol)) return fail(h, FFH_ERR_INVALID_ARG, "tol must be finite and >= 0");
   if (h->opt.dtype == FFH_BF16 && (n % 8 || m % 8))
     return fail(h, FFH_ERR_INVALID_ARG, "bf16 rows must be 16-byte aligned: n, m multiples of 8");
-  if (h->opt.variant == FFH_FROBENIUS)
-    return fail(h, FFH_ERR_UNSUPPORTED, "the Frobenius variant is not in this build");
   if (N < std::max(n, m) && h->opt.damping == 0.f)
     return fail(h, FFH_ERR_RANK, "N = %lld < max(n, m) = %lld without damping",
                 (long long)N, (long long)std::max(n, m));
@@ -453,16 +469,40 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
     CK(launch_fill_identity(A[cur], n, n, s));
   }
   const float lam = h->opt.damping;
-  const float sB = (float)(1.0 / ((double)N * (double)n));
-  const float sA = (float)(1.0 / ((double)N * (double)m));
+  const int variant = h->opt.variant;
+  const bool frob = variant == FFH_FROBENIUS;
+  const float sB = frob ? (float)(1.0 / (double)N) : (float)(1.0 / ((double)N * (double)n));
+  const float sA = frob ? (float)(1.0 / (double)N) : (float)(1.0 / ((double)N * (double)m));
   int t_done = 0;
   std::vector<IterRecord> host_recs((size_t)iters + 2);
+  if (variant == FFH_INPUT || variant == FFH_MARGINAL) {
+    // Table 1: A = E[x x^T]; B = I (Input) or E[g g^T] (Marginal); then tr A = n
+    const float s1 = (float)(1.0 / (double)N);
+    es = gram(h, xs, N, n, nullptr, s1, A[cur], partial, gtn, st);
+    if (es) return es;
+    if (variant == FFH_MARGINAL) {
+      es = gram(h, gs, N, m, nullptr, s1, B[cur], partial, gtm, st);
+      if (es) return es;
+    } else {
+      CK(launch_fill_identity(B[cur], m, m, s));
+    }
+    CK(launch_damp(A[cur], n, n, lam, st, s));
+    CK(launch_damp(B[cur], m, m, lam, st, s));
+    CK(launch_normalize(A[cur], n, B[cur], m, recs + 1, st, s));
+    iters = 0;  // no alternating loop
+    t_done = 1;
+  }
   for (int t = 1; t <= iters; ++t) {
     IterRecord* R = recs + t;
     const int nxt = cur ^ 1;
-    // ---- weights q_k = x_k^T A_{t-1}^-1 x_k
+    // ---- weights q_k = x_k^T A_{t-1}^-1 x_k  (Frobenius: x_k^T A_{t-1} x_k)
     if (t == 1 && !init) {
       CK(launch_rowsumsq(xs.raw, dtype, N, n, xs.ld_raw, q, s));
+    } else if (frob) {
+      es = chol(h, A[cur], n, L, nullptr, work, DI, st, 0);
+      if (es) return es;
+      es = qform_fwd(h, xs, N, n, L, A[cur], Mb, q, st);
+      if (es) return es;
     } else {
       es = chol(h, A[cur], n, L, Linv, work, DI, st, 0);
       if (es) return es;
@@ -477,17 +517,29 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
     // ---- B-update
     es = gram(h, gs, N, m, q, sB, B[nxt], partial, gtm, st);
     if (es) return es;
+    if (frob) {
+      CK(launch_frob2(A[cur], n, trb + 4, s));
+      CK(launch_scale_by_inv(B[nxt], m, trb + 4, s));
+    }
     CK(launch_damp(B[nxt], m, m, lam, st, s));
-    es = chol(h, B[nxt], m, L, Linv, work, DI, st,
+    es = chol(h, B[nxt], m, L, frob ? nullptr : Linv, work, DI, st,
               (t == 1 && h->opt.fault == FFH_FAULT_BAD_PIVOT) ? FFH_FAULT_BAD_PIVOT : 0);
     if (es) return es;
     CK(cudaMemcpyAsync(&R->logdet_B, &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
-    es = qform(h, gs, N, m, Linv, Mb, r, st);
+    if (frob) {
+      es = qform_fwd(h, gs, N, m, L, B[nxt], Mb, r, st);
+    } else {
+      es = qform(h, gs, N, m, Linv, Mb, r, st);
+    }
     if (es) return es;
     CK(launch_dot(q, r, N, &R->sum_qr_B, s));
     // ---- A-update
     es = gram(h, xs, N, n, r, sA, A[nxt], partial, gtn, st);
     if (es) return es;
+    if (frob) {
+      CK(launch_frob2(B[nxt], m, trb + 5, s));
+      CK(launch_scale_by_inv(A[nxt], n, trb + 5, s));
+    }
     CK(launch_damp(A[nxt], n, n, lam, st, s));
     CK(launch_normalize(A[nxt], n, B[nxt], m, R, st, s));
     // ---- convergence statistics
@@ -511,7 +563,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
       if (std::max(dA, dB) < (double)tol) break;
     }
   }
-  if (h->opt.final_loglik) {
+  if (h->opt.final_loglik && variant == FFH_FLIPFLOP) {
     es = chol(h, A[cur], n, L, Linv, work, DI, st, 0);
     if (es) return es;
     CK(cudaMemcpyAsync(&recs[t_done].logdet_A, &st->logdet, sizeof(double),
@@ -531,6 +583,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
   h->m = m;
   h->final_loglik = h->opt.final_loglik != 0;
   h->recs = host_recs;
+  h->loglik_valid = variant == FFH_FLIPFLOP;
   return es;
 }
 
@@ -743,6 +796,7 @@ extern "C" ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_
   h->m = m;
   h->final_loglik = h->opt.final_loglik != 0;
   h->recs = host_recs;
+  h->loglik_valid = true;
   return es;
 }
 
@@ -768,9 +822,11 @@ extern "C" ffh_status ffh_get_stats(ffh_t h, int32_t* iters_done, double* delta,
     const IterRecord& R = h->recs[t];
     const int i0 = 2 * (t - 1), i1 = i0 + 1;
     // l(A_{t-1}, B_t): B_t before the rescale, r computed with it
-    const double lB = -0.5 * (N * m * R.logdet_A_prev + N * n * R.logdet_B + R.sum_qr_B);
+    const double lB = h->loglik_valid
+                          ? -0.5 * (N * m * R.logdet_A_prev + N * n * R.logdet_B + R.sum_qr_B)
+                          : NAN;
     // l(A_t, B_t) after the rescale s: log|sB| = log|B| + m log s, r/s
-    const bool haveA = t < T || h->final_loglik;
+    const bool haveA = (t < T || h->final_loglik) && h->loglik_valid;
     const double ldB_s = R.logdet_B + m * std::log(R.scale);
     const double lA = haveA ? -0.5 * (N * m * R.logdet_A + N * n * ldB_s + R.sum_qr_A / R.scale)
                             : NAN;
@@ -779,7 +835,7 @@ extern "C" ffh_status ffh_get_stats(ffh_t h, int32_t* iters_done, double* delta,
       if (i1 < capacity) loglik_trace[i1] = lA;
     }
     if (mean_qr) {
-      if (i0 < capacity) mean_qr[i0] = R.sum_qr_B / N;
+      if (i0 < capacity) mean_qr[i0] = h->loglik_valid ? R.sum_qr_B / N : NAN;
       if (i1 < capacity) mean_qr[i1] = haveA ? R.sum_qr_A / (N * R.scale) : NAN;
     }
   }
@@ -943,5 +999,79 @@ extern "C" ffh_status ffh_get_timings(ffh_t h, ffh_timings* out, int32_t reset) 
       h->prof_n[k] = 0;
     }
   }
+  return FFH_OK;
+}
+
+extern "C" ffh_status ffh_phi_tilde(ffh_t h, const void* X, const void* G, int64_t N, int64_t n,
+                                    int64_t m, const float* A, const float* B, double* phi_out) {
+  if (!h) return FFH_ERR_INVALID_ARG;
+  h->err.clear();
+  ffh_status vs = validate_opt(h);
+  if (vs) return vs;
+  if (!X || !G || !A || !B || !phi_out || N < 1 || n < 1 || m < 1)
+    return fail(h, FFH_ERR_INVALID_ARG, "bad arguments");
+  if (!is_device_ptr(X) || !is_device_ptr(G) || !is_device_ptr(A) || !is_device_ptr(B))
+    return fail(h, FFH_ERR_INVALID_ARG, "ffh_phi_tilde takes device pointers");
+  const int dtype = h->opt.dtype;
+  if (dtype == FFH_BF16 && (n % 8 || m % 8))
+    return fail(h, FFH_ERR_INVALID_ARG, "bf16 rows must be 16-byte aligned: n, m multiples of 8");
+  const bool tc = h->opt.kernel == 0;
+  const int64_t D = std::max(n, m);
+  const int64_t Npad = (N + 63) / 64 * 64 + 64;
+  const int nt = (int)((D + 63) / 64);
+  auto layout = [&](Carve& c, DevStatus** st, __nv_bfloat16** Xb, __nv_bfloat16** Gb, float** q,
+                    float** r, float** L, float** Linv, __nv_bfloat16** Mb, float** work,
+                    float** DI, double** acc) {
+    *st = c.take<DevStatus>(1);
+    *Xb = (tc && dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(n)) : nullptr;
+    *Gb = (tc && dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(m)) : nullptr;
+    *q = c.take<float>(Npad);
+    *r = c.take<float>(Npad);
+    *L = c.take<float>((size_t)D * D);
+    *Linv = c.take<float>((size_t)D * D);
+    *Mb = c.take<__nv_bfloat16>((size_t)D * pad8(D));
+    *work = c.take<float>(std::max(cholesky_work_floats(D), cholesky_tc_work_bytes(D) / 4 + 1));
+    *DI = c.take<float>((size_t)nt * 64 * 64);
+    *acc = c.take<double>(4);
+  };
+  DevStatus* st;
+  __nv_bfloat16 *Xb, *Gb, *Mb;
+  float *q, *r, *L, *Linv, *work, *DI;
+  double* acc;
+  {
+    Carve c(nullptr);
+    layout(c, &st, &Xb, &Gb, &q, &r, &L, &Linv, &Mb, &work, &DI, &acc);
+    ffh_status es = ensure_ws(h, c.off + 1024);
+    if (es) return es;
+  }
+  Carve c(h->ws);
+  layout(c, &st, &Xb, &Gb, &q, &r, &L, &Linv, &Mb, &work, &DI, &acc);
+  cudaStream_t s = h->stream;
+  CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
+  Staged xs, gs;
+  ffh_status es = stage_input(h, X, true, N, n, Xb, nullptr, &xs);
+  if (es) return es;
+  es = stage_input(h, G, true, N, m, Gb, nullptr, &gs);
+  if (es) return es;
+  double ld[2] = {0, 0};
+  es = chol(h, A, n, L, Linv, work, DI, st, 0);
+  if (es) return es;
+  CK(cudaMemcpyAsync(&acc[1], &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
+  es = qform(h, xs, N, n, Linv, Mb, q, st);
+  if (es) return es;
+  es = chol(h, B, m, L, Linv, work, DI, st, 0);
+  if (es) return es;
+  CK(cudaMemcpyAsync(&acc[2], &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
+  es = qform(h, gs, N, m, Linv, Mb, r, st);
+  if (es) return es;
+  CK(launch_dot(q, r, N, &acc[0], s));
+  double hacc[3];
+  CK(cudaMemcpyAsync(hacc, acc, sizeof(hacc), cudaMemcpyDeviceToHost, s));
+  es = read_status(h, st);
+  if (es) return es;
+  (void)ld;
+  const double mean_qr = hacc[0] / (double)N;
+  *phi_out = std::exp(hacc[1] / (double)n + hacc[2] / (double)m +
+                      std::log(mean_qr / ((double)m * (double)n)));
   return FFH_OK;
 }

@@ -80,7 +80,10 @@ cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t
 // q_k = ||M v_k||^2, V bf16 N x d (pitch ld), M bf16 d x d lower (pitch ldm)
 cudaError_t launch_qform_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t ld,
                             const __nv_bfloat16* M, int64_t ldm, float* q, DevStatus* st,
-                            cudaStream_t s);
+                            cudaStream_t s, bool upper = false);
+// fp32 -> bf16 of the transpose of a lower-triangular matrix (upper result, zeros below)
+cudaError_t launch_lowerT_to_bf16(const float* src, int64_t d, int64_t lds, __nv_bfloat16* dst,
+                                  int64_t ldd, cudaStream_t s);
 size_t gram_tile_table_bytes(int64_t d);
 void gram_build_tiles(int64_t d, int2* tiles_host, int* lut_host, int* T_out);
 

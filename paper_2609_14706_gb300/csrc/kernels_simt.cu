@@ -125,6 +125,33 @@ cudaError_t launch_lower_to_bf16(const float* src, int64_t d, int64_t lds, __nv_
   return launch_to_bf16_ex(src, d, d, lds, dst, ldd, 1, s);
 }
 
+// dst[r][c] = src[c][r] for c >= r (the transpose of a lower-triangular src), 0 below;
+// 32 x 32 tiles through shared memory
+__global__ void k_lowerT_to_bf16(const float* __restrict__ src, int64_t d, int64_t lds,
+                                 __nv_bfloat16* __restrict__ dst, int64_t ldd) {
+  __shared__ float t[32][33];
+  const int64_t bx = (int64_t)blockIdx.x * 32, by = (int64_t)blockIdx.y * 32;
+  for (int r = threadIdx.y; r < 32; r += 8) {
+    const int64_t sr = by + r, sc = bx + threadIdx.x;  // source row sr, column sc
+    t[r][threadIdx.x] = (sr < d && sc < d && sc <= sr) ? src[sr * lds + sc] : 0.f;
+  }
+  __syncthreads();
+  for (int r = threadIdx.y; r < 32; r += 8) {
+    const int64_t dr = bx + r, dc = by + threadIdx.x;  // dst row = source column
+    if (dr < ldd && dc < ldd && dr < d + 8) {
+      if (dr < d) dst[dr * ldd + dc] = __float2bfloat16_rn(dc < d ? t[threadIdx.x][r] : 0.f);
+    }
+  }
+}
+
+cudaError_t launch_lowerT_to_bf16(const float* src, int64_t d, int64_t lds, __nv_bfloat16* dst,
+                                  int64_t ldd, cudaStream_t s) {
+  const unsigned nb = (unsigned)((ldd + 31) / 32);
+  k_lowerT_to_bf16<<<dim3(nb, nb), dim3(32, 8), 0, s>>>(src, d, lds, dst, ldd);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
 // ---------------------------------------------------------------------------
 // tiled fp32 GEMM (64 x 64 tiles, 256 threads, 4 x 4 per thread), batched over z:
 //   C = alpha * A * op(B) + beta * C,  op(B) = B (K x N) or B^T (B is N x K)

@@ -13,7 +13,9 @@
 //  * k_qform_tc  -- q_k = ||M v_k||^2 for lower-triangular M = L^-1 (the x^T A^-1 x of
 //                   Section 5).  Y = V M^T is formed tile by tile in TMEM and squared and
 //                   row-summed by the epilogue straight from TMEM, so Y never reaches
-//                   HBM.  Column block c of Y only needs K < 256 (c+1) (M is lower).
+//                   HBM.  Column block c of Y only needs K < 256 (c+1) (M is lower); an
+//                   upper-triangular M (the Frobenius variant's x^T A x = ||L^T x||^2)
+//                   needs K >= 256 c only.
 //
 // Both are persistent (one CTA per SM, warp-specialised): warp 0 issues TMA, warp 1
 // issues tcgen05.mma, warp 2 owns the TMEM allocation, warps 4-7 stage / drain.
@@ -456,6 +458,7 @@ constexpr int THREADS = 256;
 struct QformArgs {
   float* q;
   int64_t N;
+  int upper;  // M upper-triangular (column block c needs K >= 256 c) instead of lower
   int RB;    // row blocks
   int NC;    // column blocks
   int KBd;   // 64-wide K blocks of d
@@ -518,8 +521,9 @@ __global__ void __launch_bounds__(qf::THREADS, 1)
       bool ok = true;
       for (int rb = blockIdx.x; rb < a.RB && ok; rb += gridDim.x) {
         for (int c = 0; c < a.NC && ok; ++c) {
-          const int nk = min(a.KBd, 4 * (c + 1));
-          for (int kb = 0; kb < nk; ++kb, ++it) {
+          const int kb_lo = a.upper ? 4 * c : 0;
+          const int kb_hi = a.upper ? a.KBd : min(a.KBd, 4 * (c + 1));
+          for (int kb = kb_lo; kb < kb_hi; ++kb, ++it) {
             const int s = it % STAGES;
             const uint32_t ph = (it / STAGES) & 1;
             if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, budget)) {
@@ -556,8 +560,9 @@ __global__ void __launch_bounds__(qf::THREADS, 1)
             break;
           }
           tc_fence_after();
-          const int nk = min(a.KBd, 4 * (c + 1));
-          for (int kb = 0; kb < nk; ++kb, ++it) {
+          const int kb_lo = a.upper ? 4 * c : 0;
+          const int kb_hi = a.upper ? a.KBd : min(a.KBd, 4 * (c + 1));
+          for (int kb = kb_lo; kb < kb_hi; ++kb, ++it) {
             const int s = it % STAGES;
             const uint32_t ph = (it / STAGES) & 1;
             if (!mbar_wait(&full[s], ph, abort_flag, budget)) {
@@ -573,7 +578,7 @@ __global__ void __launch_bounds__(qf::THREADS, 1)
               // 16 K-elements = 32 B along the row.
               const uint64_t ad = sw128_desc(sa + k * 32, 16, 1024);
               const uint64_t bd = sw128_desc(sb + k * 32, 16, 1024);
-              mma_bf16(tmem + buf * BN, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+              mma_bf16(tmem + buf * BN, ad, bd, idesc, (kb > kb_lo || k > 0) ? 1u : 0u);
             }
             mma_commit(&empty[s]);
           }
@@ -632,7 +637,7 @@ __global__ void __launch_bounds__(qf::THREADS, 1)
 
 cudaError_t launch_qform_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t ld,
                             const __nv_bfloat16* M, int64_t ldm, float* q, DevStatus* st,
-                            cudaStream_t s) {
+                            cudaStream_t s, bool upper) {
   CUtensorMap vmap, mmap;
   if (!make_map_bf16(&vmap, V, (uint64_t)d, (uint64_t)N, (uint64_t)ld, qf::BK, qf::BM))
     return cudaErrorInvalidValue;
@@ -648,6 +653,7 @@ cudaError_t launch_qform_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_
   QformArgs a;
   a.q = q;
   a.N = N;
+  a.upper = upper ? 1 : 0;
   a.RB = (int)((N + qf::BM - 1) / qf::BM);
   a.NC = (int)((d + qf::BN - 1) / qf::BN);
   a.KBd = (int)((d + qf::BK - 1) / qf::BK);

@@ -303,3 +303,50 @@ def test_fit_matrix_host_input_and_damping():
         A, B = h.fit_matrix(Gk.cpu(), iters=3)
     ref = oracle.flipflop_fit_matrix(Gk.cpu(), iters=3, damping=0.1)
     assert oracle.kron_rel_err(A, B, ref.A, ref.B) <= 2e-3
+
+
+# ---------------------------------------------------------------------------
+# Table 1 variants and the mismatch factor
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("kernel", KERNELS)
+@pytest.mark.parametrize("case", ["tiny_64", "llama_small"])
+def test_frobenius_fit_matches_oracle(case, kernel):
+    wl = FIT_CASES[case].with_(iters=3)
+    X, G = synth.rank_one_samples(wl, seed=0, device="cuda")
+    with ffh.Handle(dtype=wl.dtype, kernel=kernel, variant="frobenius") as h:
+        A, B = h.fit(X, G, iters=wl.iters)
+        st = h.stats()
+    ref = oracle.frobenius_fit(X.cpu(), G.cpu(), iters=wl.iters)
+    assert oracle.kron_rel_err(A.cpu(), B.cpu(), ref.A, ref.B) <= 2e-3
+    assert np.trace(oracle.as_f64(A)) == pytest.approx(wl.n, rel=1e-4)
+    assert all(math.isnan(v) for v in st["loglik"])
+
+
+@pytest.mark.parametrize("variant", ["input", "marginal"])
+def test_input_and_marginal_hessians(variant):
+    wl = FIT_CASES["llama_small"]
+    X, G = synth.rank_one_samples(wl, seed=0, device="cuda")
+    with ffh.Handle(dtype="bf16", variant=variant) as h:
+        A, B = h.fit(X, G, iters=5)
+        st = h.stats()
+    if variant == "input":
+        Ar, Br = oracle.input_hessian(X.cpu(), wl.m)
+    else:
+        Ar, Br = oracle.marginal_hessian(X.cpu(), G.cpu())
+    assert oracle.kron_rel_err(A.cpu(), B.cpu(), Ar, Br) <= 2e-3
+    assert st["iters_done"] == 1
+
+
+def test_phi_tilde_matches_oracle_and_orders_variants():
+    """Phi~ (Section 4 mismatch factor, sample form) of the four Table 1 Hessians: the
+    GPU value matches the oracle's, and the FlipFlop fit has the smallest."""
+    wl = FIT_CASES["llama_small"].with_(iters=6)
+    X, G = synth.rank_one_samples(wl, seed=0, device="cuda")
+    phis = {}
+    for variant in ("flipflop", "frobenius", "input", "marginal"):
+        with ffh.Handle(dtype="bf16", variant=variant) as h:
+            A, B = h.fit(X, G, iters=wl.iters)
+            phis[variant] = h.phi_tilde(X, G, A, B)
+        ref = oracle.phi_tilde(X.cpu(), G.cpu(), A.cpu(), B.cpu())
+        assert math.log(phis[variant]) == pytest.approx(math.log(ref), abs=2e-3), variant
+    assert phis["flipflop"] <= min(phis["frobenius"], phis["input"], phis["marginal"]) * (1 + 1e-3)
