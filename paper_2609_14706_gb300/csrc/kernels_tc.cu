@@ -459,6 +459,8 @@ struct QformArgs {
   float* q;
   int64_t N;
   int upper;  // M upper-triangular (column block c needs K >= 256 c) instead of lower
+  int G;     // column-block groups per row block (1 or 2): with 2, two CTAs share a row
+             // block (halving the L2 working set) and add their partial sums into q
   int RB;    // row blocks
   int NC;    // column blocks
   int KBd;   // 64-wide K blocks of d
@@ -519,8 +521,10 @@ __global__ void __launch_bounds__(qf::THREADS, 1)
     if (lane == 0) {
       uint32_t it = 0;
       bool ok = true;
-      for (int rb = blockIdx.x; rb < a.RB && ok; rb += gridDim.x) {
+      for (int u = blockIdx.x; u < a.RB * a.G && ok; u += gridDim.x) {
+        const int rb = u / a.G, grp = u - rb * a.G;
         for (int c = 0; c < a.NC && ok; ++c) {
+          if (a.G == 2 && ((c + (c >> 1)) & 1) != grp) continue;
           const int kb_lo = a.upper ? 4 * c : 0;
           const int kb_hi = a.upper ? a.KBd : min(a.KBd, 4 * (c + 1));
           for (int kb = kb_lo; kb < kb_hi; ++kb, ++it) {
@@ -552,8 +556,10 @@ __global__ void __launch_bounds__(qf::THREADS, 1)
       constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, false, false);
       uint32_t it = 0, cc = 0;
       bool ok = true;
-      for (int rb = blockIdx.x; rb < a.RB && ok; rb += gridDim.x) {
-        for (int c = 0; c < a.NC; ++c, ++cc) {
+      for (int u = blockIdx.x; u < a.RB * a.G && ok; u += gridDim.x) {
+        const int grp = u % a.G;
+        for (int c = 0; c < a.NC; ++c) {
+          if (a.G == 2 && ((c + (c >> 1)) & 1) != grp) continue;
           const int buf = cc & 1;
           if (!mbar_wait(&acce[buf], ((cc >> 1) & 1) ^ 1, abort_flag, budget)) {
             ok = false;
@@ -584,6 +590,7 @@ __global__ void __launch_bounds__(qf::THREADS, 1)
           }
           if (!ok) break;
           mma_commit(&accf[buf]);
+          ++cc;
         }
       }
       if (!ok) {
@@ -598,11 +605,15 @@ __global__ void __launch_bounds__(qf::THREADS, 1)
     const int wq = warp - 4;
     uint32_t cc = 0;
     bool ok = true;
-    for (int rb = blockIdx.x; rb < a.RB && ok; rb += gridDim.x) {
+    for (int u = blockIdx.x; u < a.RB * a.G && ok; u += gridDim.x) {
+      const int rb = u / a.G, grp = u - rb * a.G;
       float acc = 0.f;
-      for (int c = 0; c < a.NC; ++c, ++cc) {
+      for (int c = 0; c < a.NC; ++c) {
+        if (a.G == 2 && ((c + (c >> 1)) & 1) != grp) continue;
         const int buf = cc & 1;
-        if (!mbar_wait(&accf[buf], (cc >> 1) & 1, abort_flag, budget)) {
+        const uint32_t aph = (cc >> 1) & 1;
+        ++cc;
+        if (!mbar_wait(&accf[buf], aph, abort_flag, budget)) {
           ok = false;
           break;
         }
@@ -619,7 +630,13 @@ __global__ void __launch_bounds__(qf::THREADS, 1)
       }
       if (!ok) break;
       const int64_t row = (int64_t)rb * BM + wq * 32 + lane;
-      if (row < a.N) a.q[row] = acc;
+      // two groups: q was zeroed and receives exactly two addends (order-independent)
+      if (row < a.N) {
+        if (a.G == 2)
+          atomicAdd(&a.q[row], acc);
+        else
+          a.q[row] = acc;
+      }
     }
     if (!ok) {
       *abort_flag = 1;
@@ -656,10 +673,15 @@ cudaError_t launch_qform_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_
   a.upper = upper ? 1 : 0;
   a.RB = (int)((N + qf::BM - 1) / qf::BM);
   a.NC = (int)((d + qf::BN - 1) / qf::BN);
+  a.G = a.NC >= 4 ? 2 : 1;
   a.KBd = (int)((d + qf::BK - 1) / qf::BK);
   a.st = st;
   a.budget_ns = kWaitBudgetNs;
-  const int grid = std::min(a.RB, num_sms());
+  if (a.G == 2) {
+    cudaError_t e = cudaMemsetAsync(q, 0, sizeof(float) * N, s);
+    if (e != cudaSuccess) return e;
+  }
+  const int grid = std::min(a.RB * a.G, num_sms());
   k_qform_tc<<<grid, qf::THREADS, qf::SMEM_BYTES, s>>>(vmap, mmap, a); note_launches(1);
   return cudaGetLastError();
 }
