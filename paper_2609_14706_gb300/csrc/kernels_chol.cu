@@ -386,101 +386,112 @@ __device__ __forceinline__ void smem_gemm(float* C, int ldc, const float* A, int
 }
 
 
-// One sub-panel sweep (Q = sub-panel index) with the panel in registers.
-// cbuf: [2][16][8] pivot-column buffer (warp-major), rbuf: [2][32] M-row buffer.
+// One sub-panel sweep (Q = sub-panel index) with the sub-panel in registers: warps 0-3
+// (named barrier 1); warp w holds rows i = w + 4 rr (rr = 0..31) of column x = c0 + lane,
+// and rows c0 + w + 4 rr (rr = 0..7) of the 32 x 32 diagonal block of the inverse.
+// cbuf: [2][4][32] pivot-column buffer (warp-major), rbuf: [2][32] M-row buffer.
+// Per pivot j the owner lane of column j has published it; every lane with x > j
+// subtracts l_ij l_xj from its column (rows above the pivot only meet entries above
+// the diagonal, which never feed entries below it and are never stored, so no row
+// predicate is needed); lanes with x <= j update the inverse rows below j.  Columns
+// and inverse rows are scaled by their pivot's 1/sqrt only at the write-back.
 template <int Q>
 __device__ __forceinline__ void leaf_sweep(float* Ls, float* Ms, float* cbuf, float* rbuf,
                                            int64_t o, DevStatus* st, bool& bad) {
   constexpr int c0 = 32 * Q;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int x = c0 + lane;
-  float a[8], m[2];
+  if (warp < 4) {
+    float a[32], m[8];
+    float my_rinv = 1.f, my_r = 1.f;
 #pragma unroll
-  for (int rr = 0; rr < 8; ++rr) {
-    const int i = warp + 16 * rr;
-    a[rr] = (i >= c0 && x <= i) ? Ls[i * LP + x] : 0.f;
-  }
+    for (int rr = 0; rr < 32; ++rr) {
+      const int i = warp + 4 * rr;
+      a[rr] = (i >= c0 && x <= i) ? Ls[i * LP + x] : 0.f;
+    }
 #pragma unroll
-  for (int rr = 0; rr < 2; ++rr) m[rr] = (c0 + warp + 16 * rr == x) ? 1.f : 0.f;
-  // publish column c0 (lane 0 of each warp) and row c0 of M (warp 0)
-  if (lane == 0) {
+    for (int rr = 0; rr < 8; ++rr) m[rr] = (c0 + warp + 4 * rr == x) ? 1.f : 0.f;
+    // publish column c0 (lane 0 of each warp) and row c0 of M (warp 0)
+    if (lane == 0) {
 #pragma unroll
-    for (int rr = 0; rr < 8; ++rr) cbuf[warp * 8 + rr] = a[rr];
-  }
-  if (warp == 0) rbuf[lane] = m[0];
-  __syncthreads();
+      for (int rr = 0; rr < 32; rr += 4)
+        *reinterpret_cast<float4*>(cbuf + warp * 32 + rr) =
+            make_float4(a[rr], a[rr + 1], a[rr + 2], a[rr + 3]);
+    }
+    if (warp == 0) rbuf[lane] = m[0];
+    asm volatile("bar.sync 1, 128;" ::: "memory");
 #pragma unroll 1
-  for (int jj = 0; jj < 32; ++jj) {
-    const int j = c0 + jj;
-    const float* cb = cbuf + (jj & 1) * 128;
-    const float* rb = rbuf + (jj & 1) * 32;
-    float* cbn = cbuf + ((jj + 1) & 1) * 128;
-    float* rbn = rbuf + ((jj + 1) & 1) * 32;
-    float ajj = cb[(j & 15) * 8 + (j >> 4)];
-    if (!(ajj > 0.f) || !isfinite(ajj)) {
-      if (tid == 0 && !bad) raise_error(st, FFH_ERR_NOT_SPD, (int)(o + j));
-      bad = true;
-      ajj = 1.f;
-    }
-    // 1/sqrt to within 2 ulp; far below the fp32 accumulation error of the update
-    const float rinv = rsqrtf(ajj);
-    const float r = ajj * rinv;
-    const float4 c_lo = *reinterpret_cast<const float4*>(cb + warp * 8);
-    const float4 c_hi = *reinterpret_cast<const float4*>(cb + warp * 8 + 4);
-    const float cv[8] = {c_lo.x, c_lo.y, c_lo.z, c_lo.w, c_hi.x, c_hi.y, c_hi.z, c_hi.w};
-    if (x > j) {
-      const float lxj = cb[(x & 15) * 8 + (x >> 4)] * rinv;
-#pragma unroll
-      for (int rr = 0; rr < 8; ++rr) {
-        const int i = warp + 16 * rr;
-        if (i > j && x <= i) a[rr] = fmaf(-cv[rr] * rinv, lxj, a[rr]);
+    for (int jj = 0; jj < 32; ++jj) {
+      const int j = c0 + jj;
+      const float* cb = cbuf + (jj & 1) * 128;
+      const float* rb = rbuf + (jj & 1) * 32;
+      float* cbn = cbuf + ((jj + 1) & 1) * 128;
+      float* rbn = rbuf + ((jj + 1) & 1) * 32;
+      float ajj = cb[(j & 3) * 32 + (j >> 2)];
+      if (!(ajj > 0.f) || !isfinite(ajj)) {
+        if (tid == 0 && !bad) raise_error(st, FFH_ERR_NOT_SPD, (int)(o + j));
+        bad = true;
+        ajj = 1.f;
       }
-    } else {
-      const float mjx = rb[lane] * rinv;
-#pragma unroll
-      for (int rr = 0; rr < 2; ++rr) {
-        const int i = c0 + warp + 16 * rr;
-        if (i > j) m[rr] = fmaf(-cv[2 * Q + rr] * rinv, mjx, m[rr]);
+      // 1/sqrt to within 2 ulp; far below the fp32 accumulation error of the update
+      const float rinv = rsqrtf(ajj);
+      if (x == j) {
+        my_rinv = rinv;
+        my_r = ajj * rinv;
       }
-    }
-    // the owner of column j scales it (pivot -> r)
-    if (x == j) {
+      float cv[32];
 #pragma unroll
-      for (int rr = 0; rr < 8; ++rr) {
-        const int i = warp + 16 * rr;
-        if (i == j)
-          a[rr] = r;
-        else if (i > j)
-          a[rr] *= rinv;
+      for (int rr = 0; rr < 32; rr += 4) {
+        const float4 t = *reinterpret_cast<const float4*>(cb + warp * 32 + rr);
+        cv[rr] = t.x;
+        cv[rr + 1] = t.y;
+        cv[rr + 2] = t.z;
+        cv[rr + 3] = t.w;
       }
-    }
-    // the owner of row j of M scales it
-    if ((j & 15) == warp && x <= j) {
-      if (jj < 16)
-        m[0] *= rinv;
-      else
-        m[1] *= rinv;
-    }
-    // publish column j+1 of L and row j+1 of M for the next pivot
-    if (jj + 1 < 32) {
-      if (x == j + 1) {
-        *reinterpret_cast<float4*>(cbn + warp * 8) = make_float4(a[0], a[1], a[2], a[3]);
-        *reinterpret_cast<float4*>(cbn + warp * 8 + 4) = make_float4(a[4], a[5], a[6], a[7]);
+      if (x > j) {
+        const float lxj = cb[(x & 3) * 32 + (x >> 2)] * rinv * rinv;
+#pragma unroll
+        for (int rr = 0; rr < 32; ++rr) a[rr] = fmaf(-cv[rr], lxj, a[rr]);
+      } else {
+        const float mjx = rb[lane] * rinv * rinv;
+#pragma unroll
+        for (int rr = 0; rr < 8; ++rr) {
+          const int i = c0 + warp + 4 * rr;
+          if (i > j) m[rr] = fmaf(-cv[8 * Q + rr], mjx, m[rr]);
+        }
       }
-      if (((j + 1) & 15) == warp) rbn[lane] = (jj + 1 < 16) ? m[0] : m[1];
+      // publish column j+1 (its owner lane) and row j+1 of M (its owner warp)
+      if (jj + 1 < 32) {
+        if (x == j + 1) {
+#pragma unroll
+          for (int rr = 0; rr < 32; rr += 4)
+            *reinterpret_cast<float4*>(cbn + warp * 32 + rr) =
+                make_float4(a[rr], a[rr + 1], a[rr + 2], a[rr + 3]);
+        }
+        if (((j + 1) & 3) == warp) {
+          const int rm = (jj + 1) >> 2;
+          float v = m[0];
+#pragma unroll
+          for (int rr = 1; rr < 8; ++rr)
+            if (rr == rm) v = m[rr];
+          rbn[lane] = v;
+        }
+      }
+      asm volatile("bar.sync 1, 128;" ::: "memory");
     }
-    __syncthreads();
-  }
-  // write the finished sub-panel and the diagonal block of the inverse back
+    // write back, scaling column x by its pivot's 1/sqrt (the pivot itself -> sqrt) and
+    // row i of the inverse by pivot i's 1/sqrt (held by lane i - c0)
 #pragma unroll
-  for (int rr = 0; rr < 8; ++rr) {
-    const int i = warp + 16 * rr;
-    if (i >= c0 && x <= i) Ls[i * LP + x] = a[rr];
-  }
+    for (int rr = 0; rr < 32; ++rr) {
+      const int i = warp + 4 * rr;
+      if (i >= c0 && x <= i) Ls[i * LP + x] = (i == x) ? my_r : a[rr] * my_rinv;
+    }
 #pragma unroll
-  for (int rr = 0; rr < 2; ++rr) {
-    const int i = c0 + warp + 16 * rr;
-    Ms[i * LP + x] = (x <= i) ? m[rr] : 0.f;
+    for (int rr = 0; rr < 8; ++rr) {
+      const int i = c0 + warp + 4 * rr;
+      const float ri = __shfl_sync(0xffffffffu, my_rinv, i - c0);
+      Ms[i * LP + x] = (x <= i) ? m[rr] * ri : 0.f;
+    }
   }
   __syncthreads();
 }
@@ -525,7 +536,7 @@ __global__ void __launch_bounds__(LEAF_THREADS) k_chol_leaf(float* W, int64_t ld
   __syncthreads();
   float ld_acc = 0.f;
   bool bad = false;
-  float* cbuf = Ts;        // [2][16][8]  (Ts is free until the doubling)
+  float* cbuf = Ts;        // [2][4][32]  (Ts is free until the doubling)
   float* rbuf = Ts + 256;  // [2][32]
 #pragma unroll 1
   for (int q = 0; q < LB / 32; ++q) {
@@ -590,18 +601,41 @@ __global__ void __launch_bounds__(LEAF_THREADS) k_chol_leaf(float* W, int64_t ld
   smem_gemm<64>(Ms + 64 * LP, LP, Ms + 64 * LP + 64, LP, Ts, 65, 0, 64, -1.f, false, tid,
                 LEAF_THREADS);
   __syncthreads();
-  for (int idx = tid; idx < LB * LB; idx += LEAF_THREADS) {
-    const int i = idx >> 7, j = idx & 127;
-    const float mv = (j <= i) ? Ms[i * LP + j] : 0.f;
-    if (i < b && j < b) {
-      L[(o + i) * ldl + (o + j)] = (j <= i) ? Ls[i * LP + j] : 0.f;
-      Minv[(o + i) * ldm + (o + j)] = mv;
+  // write-out, four consecutive columns per thread
+  const bool vec_ok = ((ldl | ldm) & 3) == 0 && (o & 3) == 0 &&
+                      ((reinterpret_cast<uintptr_t>(L) | reinterpret_cast<uintptr_t>(Minv)) & 15) == 0;
+  for (int idx = tid; idx < LB * LB / 4; idx += LEAF_THREADS) {
+    const int i = idx >> 5, j0 = (idx & 31) * 4;
+    float lv[4], mv[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int j = j0 + e;
+      lv[e] = (j <= i) ? Ls[i * LP + j] : 0.f;
+      mv[e] = (j <= i && i < b && j < b) ? Ms[i * LP + j] : 0.f;
+    }
+    if (i < b) {
+      if (vec_ok && j0 + 3 < b) {
+        *reinterpret_cast<float4*>(L + (o + i) * ldl + o + j0) = make_float4(lv[0], lv[1], lv[2], lv[3]);
+        *reinterpret_cast<float4*>(Minv + (o + i) * ldm + o + j0) =
+            make_float4(mv[0], mv[1], mv[2], mv[3]);
+      } else {
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          if (j0 + e < b) {
+            L[(o + i) * ldl + o + j0 + e] = lv[e];
+            Minv[(o + i) * ldm + o + j0 + e] = mv[e];
+          }
+      }
     }
     if (m11_split) {
-      const float xx = (i < b && j < b) ? mv : 0.f;
-      const __nv_bfloat16 hi = __float2bfloat16_rn(xx);
-      m11_split[i * 2 * LB + j] = hi;
-      m11_split[i * 2 * LB + LB + j] = __float2bfloat16_rn(xx - __bfloat162float(hi));
+      __nv_bfloat16 hi[4], lo[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        hi[e] = __float2bfloat16_rn(mv[e]);
+        lo[e] = __float2bfloat16_rn(mv[e] - __bfloat162float(hi[e]));
+      }
+      *reinterpret_cast<uint2*>(m11_split + i * 2 * LB + j0) = *reinterpret_cast<uint2*>(hi);
+      *reinterpret_cast<uint2*>(m11_split + i * 2 * LB + LB + j0) = *reinterpret_cast<uint2*>(lo);
     }
   }
   if (tid == 0) atomicAdd(&st->logdet, 2.0 * (double)ld_acc);
