@@ -10,6 +10,7 @@ Llama-7B-like attention projection n = m = 4096, N = 262144 bf16 samples,
 flush is needed between steps.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload NAME] [--samples N]
 
 With N > 1 (torchrun, one rank per GPU) every rank fits its own layer (independent
 problems, weak scaling, no collective in the data path); rank 0 prints the line.
@@ -51,6 +52,9 @@ def parse_args():
     p.add_argument("--seed", type=int, default=0)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--samples", type=int, default=None,
+                   help="override the workload's sample count N (short profiling runs; "
+                        "the headline uses the workload's own N)")
     return p.parse_args()
 
 
@@ -221,6 +225,8 @@ def run_ours(args):
         dist_mod.init_process_group("nccl")
         dist = dist_mod
     wl = synth.WORKLOADS[args.workload]
+    if args.samples:
+        wl = wl.with_(N=args.samples)
     matrix = wl.kind == "matrix"
     iters = wl.iters
     N, n, m = wl.N, wl.n, wl.m

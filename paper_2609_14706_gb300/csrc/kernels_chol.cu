@@ -333,180 +333,159 @@ static cudaError_t split(const float* src, int64_t lds, int64_t src_stride, int 
 
 // ---------------------------------------------------------------------------
 // 128 x 128 diagonal block: Cholesky factor L11 and inverse M11 = L11^-1, one CTA of
-// 512 threads (16 warps).
-//   Four 32-column sub-panels.  During a sub-panel's sweep it lives in registers:
-//   thread (warp w, lane l) holds column x = c0 + l of rows w, w+16, ..., w+112, and of
-//   the 32 x 32 diagonal block of the inverse the rows c0+w, c0+w+16.  Pivot j needs
-//   only column j of L and row j of M from other threads: their owners publish them to a
-//   double-buffered shared array at the end of pivot j-1 (one barrier per pivot).  At
-//   pivot j, x > j: L[i][x] -= l_ij l_xj (rows i > j); x <= j: M[i][x] -= l_ij m_jx
-//   (rows j < i < c0+32), the elimination applied to the identity (forward
-//   substitution in right-looking order); the owners of column j and row j scale them
-//   by 1/sqrt(pivot).  The finished sub-panel updates the trailing lower triangle as a
-//   rank-32 product in shared memory (4 x 4 register blocks).  The 128 x 128 inverse is
-//   assembled from the four 32 x 32 blocks by doubling,
-//   [[L11,0],[L21,L22]]^-1 = [[M11,0],[-M22 (L21 M11), M22]].
+// 512 threads (16 warps), blocked by 32 (sub-panels q = 0..3, rows/cols Q = [32q, 32q+32)).
+//   A(q)  warp 0 factors the 32 x 32 diagonal block D_q and inverts it in registers:
+//         lane i holds row i of D_q and column i of its inverse; pivot j is broadcast
+//         by shuffle, and the remaining columns shift down one register per pivot so
+//         every register index is static.  Writes L_qq, Mi_q = L_qq^-1 and
+//         Mt[x][k] = Mi_q[k][x].
+//   B(q)  all warps: the rows below, L[r][Q] = A[r][Q] Mi_q^T (4 x 4 register blocks),
+//         also stored transposed, Pt[k][r] = L[r][32q+k].
+//   C(q)  warps 0-1 apply the rank-32 update of sub-panel q to D_{q+1} and warp 0 goes
+//         on to A(q+1), while warps 2-15 update the rest of the trailing lower triangle
+//         and form row block q of the inverse by block forward substitution,
+//         M[Q][0:32q] = -Mi_q (L[Q][0:32q] M[0:32q][0:32q]).
+// Pt and Mt are double-buffered by the parity of q, so A(q+1) never writes what C(q)
+// reads.  The pivot product gives log|F11| = sum_j log(pivot_j).
 // Outputs: L11 and M11 (fp32) and the bf16 hi/lo split of M11 ([hi | lo] rows, pitch
 // 256), the B operand of the panel GEMM.
 // ---------------------------------------------------------------------------
 constexpr int LB = 128;
-constexpr int LP = LB + 1;  // padded pitch
-constexpr int LB_SMEM = (2 * LB * LP + 64 * 65) * 4 + 64;
+constexpr int LP = LB + 1;   // pitch of the row-major 128 x 128 blocks (conflict-free columns)
+constexpr int PTP = LB + 4;  // pitch of Pt (float4 rows)
+constexpr int MTP = 36;      // pitch of Mt
+constexpr int TP = 100;      // pitch of the 32 x 96 scratch T
+constexpr int LB_SMEM =
+    (2 * LB * LP + 2 * 32 * PTP + 2 * 32 * MTP + 32 * TP) * 4 + 64;
 constexpr int LEAF_THREADS = 512;
 
-// C[r][c] (+)= sgn * sum_k A[r][k] B[k][c] on a 32 x 32 (or 64 x 64) block in shared
-// memory, with 4 x 4 register blocks; thread t of nthreads covers blocks t, t+nthreads.
-template <int S>
-__device__ __forceinline__ void smem_gemm(float* C, int ldc, const float* A, int lda,
-                                          const float* B, int ldb, int kbeg, int kend, float sgn,
-                                          bool accumulate, int t, int nthreads) {
-  constexpr int NB = S / 4;
-  for (int blk = t; blk < NB * NB; blk += nthreads) {
-    const int br = (blk / NB) * 4, bc = (blk % NB) * 4;
+// A(q): factor and invert the diagonal block (warp 0 only).  Returns sum log(pivot)
+// (fp32: FP64 arithmetic is slow on this part and would sit on the pivot chain).
+__device__ __forceinline__ float leaf_diag(float* Ls, float* Ms, float* Mt, int c0,
+                                            int64_t o, DevStatus* st, bool& bad) {
+  const int lane = threadIdx.x & 31;
+  constexpr unsigned FULL = 0xffffffffu;
+  float a[32], mc[32];
+#pragma unroll
+  for (int k = 0; k < 32; ++k) {
+    a[k] = (k <= lane) ? Ls[(c0 + lane) * LP + c0 + k] : 0.f;
+    mc[k] = (k == lane) ? 1.f : 0.f;
+  }
+  float lg = 0.f;
+#pragma unroll 1
+  for (int j = 0; j < 32; ++j) {
+    // registers k = 0..31 hold columns j+k of row `lane` (of D) and rows j+k of column
+    // `lane` (of the inverse)
+    float piv = __shfl_sync(FULL, a[0], j);
+    if (!(piv > 0.f) || !isfinite(piv)) {  // warp-uniform (broadcast value)
+      if (lane == 0 && !bad) raise_error(st, FFH_ERR_NOT_SPD, (int)(o + c0 + j));
+      bad = true;
+      piv = 1.f;
+    }
+    // 1/sqrt to within 2 ulp; far below the fp32 accumulation error of the updates
+    const float r = rsqrtf(piv);
+    const float l = a[0] * r;   // lane > j: l_{lane,j}; lane j: sqrt(pivot)
+    const float m = mc[0] * r;  // Mi[j][lane] (exactly 0 for lane > j)
+    lg += logf(piv);
+    Ls[(c0 + lane) * LP + c0 + j] = lane >= j ? l : 0.f;
+    Ms[(c0 + j) * LP + c0 + lane] = m;
+    Mt[lane * MTP + j] = m;
+#pragma unroll
+    for (int k = 1; k < 32; ++k) {
+      // l_{j+k, j}; for j + k > 31 the value is unused (shifted past the block)
+      const float lk = __shfl_sync(FULL, l, (j + k) & 31);
+      a[k - 1] = fmaf(-l, lk, a[k]);
+      mc[k - 1] = fmaf(-lk, m, mc[k]);
+    }
+    a[31] = 0.f;
+    mc[31] = 0.f;
+  }
+  return lg;
+}
+
+// Rank-32 update of one 4 x 4 block of the trailing lower triangle from the transposed
+// sub-panel: A[r][c] -= sum_k Pt[k][r] Pt[k][c].
+__device__ __forceinline__ void leaf_trail_block(float* Ls, const float* Pt, int r0, int cc0) {
+  float acc[4][4] = {};
+#pragma unroll 8
+  for (int k = 0; k < 32; ++k) {
+    const float4 av = *reinterpret_cast<const float4*>(Pt + k * PTP + r0);
+    const float4 bv = *reinterpret_cast<const float4*>(Pt + k * PTP + cc0);
+    const float ar[4] = {av.x, av.y, av.z, av.w}, br[4] = {bv.x, bv.y, bv.z, bv.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int jx = 0; jx < 4; ++jx) acc[i][jx] = fmaf(ar[i], br[jx], acc[i][jx]);
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int jx = 0; jx < 4; ++jx)
+      if (cc0 + jx <= r0 + i) Ls[(r0 + i) * LP + cc0 + jx] -= acc[i][jx];
+}
+
+// Row block q >= 1 of the inverse: T = L[Q][0:c0] M[0:c0][0:c0], then
+// M[Q][0:c0] = -Mi_q T.  Threads t = 0..nt-1; `sync` separates the two products.
+template <class Sync>
+__device__ __forceinline__ void leaf_inverse_rows(float* Ls, float* Ms, float* T, int c0, int t,
+                                                  int nt, Sync sync) {
+  const int nbx = c0 / 4;  // 4-wide column blocks of [0, c0)
+  for (int blk = t; blk < 8 * nbx; blk += nt) {
+    const int i0 = (blk / nbx) * 4, x0 = (blk % nbx) * 4;
     float acc[4][4] = {};
-    for (int k = kbeg; k < kend; ++k) {
+    // M lower triangular: M[k][x] = 0 for k < x, so k starts at x0
+    for (int k = x0; k < c0; ++k) {
       float av[4], bv[4];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) av[i] = A[(br + i) * lda + k];
+      for (int i = 0; i < 4; ++i) av[i] = Ls[(c0 + i0 + i) * LP + k];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) bv[j] = B[k * ldb + bc + j];
+      for (int jx = 0; jx < 4; ++jx) bv[jx] = Ms[k * LP + x0 + jx];
 #pragma unroll
       for (int i = 0; i < 4; ++i)
 #pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+        for (int jx = 0; jx < 4; ++jx) acc[i][jx] = fmaf(av[i], bv[jx], acc[i][jx]);
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      *reinterpret_cast<float4*>(T + (i0 + i) * TP + x0) =
+          make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+  }
+  sync();
+  for (int blk = t; blk < 8 * nbx; blk += nt) {
+    const int i0 = (blk / nbx) * 4, x0 = (blk % nbx) * 4;
+    float acc[4][4] = {};
+    // Mi_q lower triangular: row i needs j <= i < i0 + 4
+    for (int j = 0; j < i0 + 4; ++j) {
+      float av[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) av[i] = Ms[(c0 + i0 + i) * LP + c0 + j];
+      const float4 bv = *reinterpret_cast<const float4*>(T + j * TP + x0);
+      const float br[4] = {bv.x, bv.y, bv.z, bv.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int jx = 0; jx < 4; ++jx) acc[i][jx] = fmaf(av[i], br[jx], acc[i][jx]);
     }
 #pragma unroll
     for (int i = 0; i < 4; ++i)
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        float* cp = C + (br + i) * ldc + bc + j;
-        *cp = accumulate ? fmaf(sgn, acc[i][j], *cp) : sgn * acc[i][j];
-      }
+      for (int jx = 0; jx < 4; ++jx) Ms[(c0 + i0 + i) * LP + x0 + jx] = -acc[i][jx];
   }
 }
 
-
-// One sub-panel sweep (Q = sub-panel index) with the sub-panel in registers: warps 0-3
-// (named barrier 1); warp w holds rows i = w + 4 rr (rr = 0..31) of column x = c0 + lane,
-// and rows c0 + w + 4 rr (rr = 0..7) of the 32 x 32 diagonal block of the inverse.
-// cbuf: [2][4][32] pivot-column buffer (warp-major), rbuf: [2][32] M-row buffer.
-// Per pivot j the owner lane of column j has published it; every lane with x > j
-// subtracts l_ij l_xj from its column (rows above the pivot only meet entries above
-// the diagonal, which never feed entries below it and are never stored, so no row
-// predicate is needed); lanes with x <= j update the inverse rows below j.  Columns
-// and inverse rows are scaled by their pivot's 1/sqrt only at the write-back.
-template <int Q>
-__device__ __forceinline__ void leaf_sweep(float* Ls, float* Ms, float* cbuf, float* rbuf,
-                                           int64_t o, DevStatus* st, bool& bad) {
-  constexpr int c0 = 32 * Q;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int x = c0 + lane;
-  if (warp < 4) {
-    float a[32], m[8];
-    float my_rinv = 1.f, my_r = 1.f;
-#pragma unroll
-    for (int rr = 0; rr < 32; ++rr) {
-      const int i = warp + 4 * rr;
-      a[rr] = (i >= c0 && x <= i) ? Ls[i * LP + x] : 0.f;
-    }
-#pragma unroll
-    for (int rr = 0; rr < 8; ++rr) m[rr] = (c0 + warp + 4 * rr == x) ? 1.f : 0.f;
-    // publish column c0 (lane 0 of each warp) and row c0 of M (warp 0)
-    if (lane == 0) {
-#pragma unroll
-      for (int rr = 0; rr < 32; rr += 4)
-        *reinterpret_cast<float4*>(cbuf + warp * 32 + rr) =
-            make_float4(a[rr], a[rr + 1], a[rr + 2], a[rr + 3]);
-    }
-    if (warp == 0) rbuf[lane] = m[0];
-    asm volatile("bar.sync 1, 128;" ::: "memory");
-#pragma unroll 1
-    for (int jj = 0; jj < 32; ++jj) {
-      const int j = c0 + jj;
-      const float* cb = cbuf + (jj & 1) * 128;
-      const float* rb = rbuf + (jj & 1) * 32;
-      float* cbn = cbuf + ((jj + 1) & 1) * 128;
-      float* rbn = rbuf + ((jj + 1) & 1) * 32;
-      float ajj = cb[(j & 3) * 32 + (j >> 2)];
-      if (!(ajj > 0.f) || !isfinite(ajj)) {
-        if (tid == 0 && !bad) raise_error(st, FFH_ERR_NOT_SPD, (int)(o + j));
-        bad = true;
-        ajj = 1.f;
-      }
-      // 1/sqrt to within 2 ulp; far below the fp32 accumulation error of the update
-      const float rinv = rsqrtf(ajj);
-      if (x == j) {
-        my_rinv = rinv;
-        my_r = ajj * rinv;
-      }
-      float cv[32];
-#pragma unroll
-      for (int rr = 0; rr < 32; rr += 4) {
-        const float4 t = *reinterpret_cast<const float4*>(cb + warp * 32 + rr);
-        cv[rr] = t.x;
-        cv[rr + 1] = t.y;
-        cv[rr + 2] = t.z;
-        cv[rr + 3] = t.w;
-      }
-      if (x > j) {
-        const float lxj = cb[(x & 3) * 32 + (x >> 2)] * rinv * rinv;
-#pragma unroll
-        for (int rr = 0; rr < 32; ++rr) a[rr] = fmaf(-cv[rr], lxj, a[rr]);
-      } else {
-        const float mjx = rb[lane] * rinv * rinv;
-#pragma unroll
-        for (int rr = 0; rr < 8; ++rr) {
-          const int i = c0 + warp + 4 * rr;
-          if (i > j) m[rr] = fmaf(-cv[8 * Q + rr], mjx, m[rr]);
-        }
-      }
-      // publish column j+1 (its owner lane) and row j+1 of M (its owner warp)
-      if (jj + 1 < 32) {
-        if (x == j + 1) {
-#pragma unroll
-          for (int rr = 0; rr < 32; rr += 4)
-            *reinterpret_cast<float4*>(cbn + warp * 32 + rr) =
-                make_float4(a[rr], a[rr + 1], a[rr + 2], a[rr + 3]);
-        }
-        if (((j + 1) & 3) == warp) {
-          const int rm = (jj + 1) >> 2;
-          float v = m[0];
-#pragma unroll
-          for (int rr = 1; rr < 8; ++rr)
-            if (rr == rm) v = m[rr];
-          rbn[lane] = v;
-        }
-      }
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-    }
-    // write back, scaling column x by its pivot's 1/sqrt (the pivot itself -> sqrt) and
-    // row i of the inverse by pivot i's 1/sqrt (held by lane i - c0)
-#pragma unroll
-    for (int rr = 0; rr < 32; ++rr) {
-      const int i = warp + 4 * rr;
-      if (i >= c0 && x <= i) Ls[i * LP + x] = (i == x) ? my_r : a[rr] * my_rinv;
-    }
-#pragma unroll
-    for (int rr = 0; rr < 8; ++rr) {
-      const int i = c0 + warp + 4 * rr;
-      const float ri = __shfl_sync(0xffffffffu, my_rinv, i - c0);
-      Ms[i * LP + x] = (x <= i) ? m[rr] * ri : 0.f;
-    }
-  }
-  __syncthreads();
-}
-
-__global__ void __launch_bounds__(LEAF_THREADS) k_chol_leaf(float* W, int64_t ldw, int64_t d,
-                                                            int64_t o, float* L, int64_t ldl,
-                                                            float* Minv, int64_t ldm,
-                                                            __nv_bfloat16* m11_split,
-                                                            DevStatus* st, int fault) {
+__global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t ldw, int64_t d,
+                                                               int64_t o, float* L, int64_t ldl,
+                                                               float* Minv, int64_t ldm,
+                                                               __nv_bfloat16* m11_split,
+                                                               DevStatus* st, int fault) {
   extern __shared__ float sh[];
-  float* Ls = sh;             // [LB][LP]
-  float* Ms = sh + LB * LP;   // [LB][LP]
-  float* Ts = sh + 2 * LB * LP;  // [64][65] temporary
+  float* Ls = sh;                      // [LB][LP]  working block -> L11
+  float* Ms = Ls + LB * LP;            // [LB][LP]  M11
+  float* Ptb = Ms + LB * LP;           // [2][32][PTP] transposed sub-panels
+  float* Mtb = Ptb + 2 * 32 * PTP;     // [2][32][MTP] transposed diagonal-block inverses
+  float* T = Mtb + 2 * 32 * MTP;       // [32][TP]
   const int b = (int)((d - o) < LB ? (d - o) : LB);
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int tid = threadIdx.x, warp = tid >> 5;
   for (int idx = tid; idx < LB * LB / 4; idx += LEAF_THREADS) {
     const int i = idx >> 5, j4 = (idx & 31) * 4;
     float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -526,7 +505,7 @@ __global__ void __launch_bounds__(LEAF_THREADS) k_chol_leaf(float* W, int64_t ld
     for (int e = 0; e < 4; ++e) {
       const int j = j4 + e;
       float x = (j <= i) ? vv[e] : 0.f;
-      if (i >= b || j >= b) x = (i == j) ? 1.f : 0.f;
+      if (i >= b || j >= b) x = (i == j) ? 1.f : 0.f;  // identity padding
       Ls[i * LP + j] = x;
       Ms[i * LP + j] = 0.f;
     }
@@ -534,73 +513,72 @@ __global__ void __launch_bounds__(LEAF_THREADS) k_chol_leaf(float* W, int64_t ld
   __syncthreads();
   if (tid == 0 && fault == FFH_FAULT_BAD_PIVOT && o == 0) Ls[0] = __int_as_float(0x7fc00000);
   __syncthreads();
-  float ld_acc = 0.f;
   bool bad = false;
-  float* cbuf = Ts;        // [2][4][32]  (Ts is free until the doubling)
-  float* rbuf = Ts + 256;  // [2][32]
+  float lg = 0.f;  // held by warp 0
+  if (warp == 0) lg += leaf_diag(Ls, Ms, Mtb, 0, o, st, bad);
+  __syncthreads();
 #pragma unroll 1
-  for (int q = 0; q < LB / 32; ++q) {
+  for (int q = 0; q < 4; ++q) {
     const int c0 = 32 * q;
-    if (q == 0) leaf_sweep<0>(Ls, Ms, cbuf, rbuf, o, st, bad);
-    if (q == 1) leaf_sweep<1>(Ls, Ms, cbuf, rbuf, o, st, bad);
-    if (q == 2) leaf_sweep<2>(Ls, Ms, cbuf, rbuf, o, st, bad);
-    if (q == 3) leaf_sweep<3>(Ls, Ms, cbuf, rbuf, o, st, bad);
-    // trailing rank-32 update of the lower triangle: A[r][c] -= sum_k L[r][c0+k] L[c][c0+k]
-    const int r0 = c0 + 32;
-    const int nb = (LB - r0) / 4;  // 4 x 4 blocks per side
-    for (int blk = tid; blk < nb * nb; blk += LEAF_THREADS) {
-      const int bi = blk / nb, bj = blk - bi * nb;
-      if (bj > bi) continue;
-      const int rr = r0 + 4 * bi, cc = r0 + 4 * bj;
-      float acc[4][4] = {};
-#pragma unroll 4
-      for (int k = 0; k < 32; ++k) {
-        float av[4], bv[4];
+    float* Pt = Ptb + (q & 1) * 32 * PTP;
+    const float* Mt = Mtb + (q & 1) * 32 * MTP;
+    // B(q): rows r in [c0 + 32, 128) of the sub-panel, L[r][c0 + k] = sum_x A[r][c0 + x] Mi[k][x].
+    // At most one 4 x 4 block per thread; results are held across a barrier because the
+    // blocks of a row read the A entries that other blocks of the row overwrite.
+    const int R = LB - c0 - 32;
+    const bool has = tid < (R / 4) * 8;
+    const int r0 = c0 + 32 + (tid >> 3) * 4, k0 = (tid & 7) * 4;
+    float acc[4][4] = {};
+    if (has) {
+      for (int x = 0; x < k0 + 4; ++x) {  // Mi[k][x] = 0 for x > k
+        float av[4];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) av[i] = Ls[(rr + i) * LP + c0 + k];
-#pragma unroll
-        for (int jx = 0; jx < 4; ++jx) bv[jx] = Ls[(cc + jx) * LP + c0 + k];
+        for (int i = 0; i < 4; ++i) av[i] = Ls[(r0 + i) * LP + c0 + x];
+        const float4 bv = *reinterpret_cast<const float4*>(Mt + x * MTP + k0);
+        const float br[4] = {bv.x, bv.y, bv.z, bv.w};
 #pragma unroll
         for (int i = 0; i < 4; ++i)
 #pragma unroll
-          for (int jx = 0; jx < 4; ++jx) acc[i][jx] = fmaf(av[i], bv[jx], acc[i][jx]);
+          for (int jx = 0; jx < 4; ++jx) acc[i][jx] = fmaf(av[i], br[jx], acc[i][jx]);
       }
+    }
+    __syncthreads();
+    if (has) {
 #pragma unroll
       for (int i = 0; i < 4; ++i)
 #pragma unroll
-        for (int jx = 0; jx < 4; ++jx)
-          if (cc + jx <= rr + i) Ls[(rr + i) * LP + cc + jx] -= acc[i][jx];
+        for (int jx = 0; jx < 4; ++jx) Ls[(r0 + i) * LP + c0 + k0 + jx] = acc[i][jx];
+#pragma unroll
+      for (int jx = 0; jx < 4; ++jx)
+        *reinterpret_cast<float4*>(Pt + (k0 + jx) * PTP + r0) =
+            make_float4(acc[0][jx], acc[1][jx], acc[2][jx], acc[3][jx]);
+    }
+    __syncthreads();
+    if (q < 3) {
+      const int nb = R / 4;  // 4-row blocks of the trailing matrix [c0 + 32, 128)
+      if (warp < 2) {
+        // D_{q+1} first (4-blocks bi, bj < 8), then warp 0 factors it
+        const int bi = tid >> 3, bj = tid & 7;
+        if (bj <= bi) leaf_trail_block(Ls, Pt, c0 + 32 + 4 * bi, c0 + 32 + 4 * bj);
+        asm volatile("bar.sync 1, 64;" ::: "memory");
+        if (warp == 0)
+          lg += leaf_diag(Ls, Ms, Mtb + ((q + 1) & 1) * 32 * MTP, c0 + 32, o, st, bad);
+      } else {
+        const int t = tid - 64;
+        for (int blk = t; blk < nb * nb; blk += LEAF_THREADS - 64) {
+          const int bi = blk / nb, bj = blk - (blk / nb) * nb;
+          if (bi < 8 || bj > bi) continue;
+          leaf_trail_block(Ls, Pt, c0 + 32 + 4 * bi, c0 + 32 + 4 * bj);
+        }
+        if (q >= 1)
+          leaf_inverse_rows(Ls, Ms, T, c0, t, LEAF_THREADS - 64,
+                            [] { asm volatile("bar.sync 2, 448;" ::: "memory"); });
+      }
+    } else {
+      leaf_inverse_rows(Ls, Ms, T, c0, tid, LEAF_THREADS, [] { __syncthreads(); });
     }
     __syncthreads();
   }
-  // log|F| of this block = 2 sum_i log L_ii
-  if (warp < 4) {
-    const int i = tid;
-    float lg = (i < b) ? logf(Ls[i * LP + i]) : 0.f;
-    for (int off = 16; off > 0; off >>= 1) lg += __shfl_down_sync(0xffffffffu, lg, off);
-    if (lane == 0) Ts[64 * 65 - 4 + warp] = lg;
-  }
-  __syncthreads();
-  if (tid == 0)
-    ld_acc = Ts[64 * 65 - 4] + Ts[64 * 65 - 3] + Ts[64 * 65 - 2] + Ts[64 * 65 - 1];
-  __syncthreads();
-  // doubling, h = 32: pairs (0,1) and (2,3); h = 64: pair (0,1)
-  {
-    // pair pr = tid / 256 (threads 0-255 take pair 0, 256-511 pair 1); T = L21 M11
-    // (32 x 32, pair pr in columns 32 pr .. of Ts), then M21 = -M22 T
-    const int pr = tid >> 8, tp = tid & 255, ob = 64 * pr;
-    smem_gemm<32>(Ts + pr * 32, 65, Ls + (ob + 32) * LP + ob, LP, Ms + ob * LP + ob, LP, 0, 32,
-                  1.f, false, tp, 256);
-    __syncthreads();
-    smem_gemm<32>(Ms + (ob + 32) * LP + ob, LP, Ms + (ob + 32) * LP + ob + 32, LP, Ts + pr * 32,
-                  65, 0, 32, -1.f, false, tp, 256);
-    __syncthreads();
-  }
-  smem_gemm<64>(Ts, 65, Ls + 64 * LP, LP, Ms, LP, 0, 64, 1.f, false, tid, LEAF_THREADS);
-  __syncthreads();
-  smem_gemm<64>(Ms + 64 * LP, LP, Ms + 64 * LP + 64, LP, Ts, 65, 0, 64, -1.f, false, tid,
-                LEAF_THREADS);
-  __syncthreads();
   // write-out, four consecutive columns per thread
   const bool vec_ok = ((ldl | ldm) & 3) == 0 && (o & 3) == 0 &&
                       ((reinterpret_cast<uintptr_t>(L) | reinterpret_cast<uintptr_t>(Minv)) & 15) == 0;
@@ -638,7 +616,7 @@ __global__ void __launch_bounds__(LEAF_THREADS) k_chol_leaf(float* W, int64_t ld
       *reinterpret_cast<uint2*>(m11_split + i * 2 * LB + LB + j0) = *reinterpret_cast<uint2*>(lo);
     }
   }
-  if (tid == 0) atomicAdd(&st->logdet, 2.0 * (double)ld_acc);
+  if (tid == 0) atomicAdd(&st->logdet, (double)lg);
 }
 
 size_t cholesky_tc_work_bytes(int64_t d) {
