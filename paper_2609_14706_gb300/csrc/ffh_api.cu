@@ -289,16 +289,27 @@ ffh_status stage_input(ffh_t h, const void* V, bool on_dev, int64_t N, int64_t d
   return FFH_OK;
 }
 
+// C = scale * V^T diag(w) V.  With a scratch `vw` (N rows of V.ld_bf bf16) the weights are
+// applied to a copy of V first and the tensor-core Gram runs unweighted on (diag(w) V, V):
+// the same bf16 operands, without the in-kernel scaling pass competing with the MMA for
+// shared-memory bandwidth.
 ffh_status gram(ffh_t h, const Staged& V, int64_t N, int64_t d, const float* w_padded, float scale,
-                float* C, float* partial, const GramTables& gt, DevStatus* st) {
+                float* C, float* partial, const GramTables& gt, DevStatus* st,
+                __nv_bfloat16* vw = nullptr) {
   cudaEvent_t t0 = prof_begin(h);
   if (h->opt.kernel == 1) {
     CK(launch_gram_simt(V.raw, h->opt.dtype, N, d, V.ld_raw, w_padded, scale, C, d, h->stream));
     prof_end(h, PROF_GRAM, t0);
   } else {
     cudaEvent_t t1 = t0 ? next_event(h) : nullptr;
+    const __nv_bfloat16* va = nullptr;
+    if (vw && w_padded) {
+      CK(launch_scale_rows(V.bf, V.ld_bf, N, d, w_padded, vw, V.ld_bf, h->stream));
+      va = vw;
+      w_padded = nullptr;
+    }
     CK(launch_gram_tc(V.bf, N, d, V.ld_bf, w_padded, scale, C, d, partial, gt.tiles, gt.lut,
-                      gt.plan, st, h->opt.fault, h->stream, t1));
+                      gt.plan, st, h->opt.fault, h->stream, t1, va, V.ld_bf));
     prof_end(h, PROF_GRAM, t0, t1);
   }
   return FFH_OK;
@@ -397,7 +408,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
                     __nv_bfloat16** Gb, float** stage, float** q, float** r, float** A2,
                     float** B2, float** L, float** Linv, __nv_bfloat16** Mb, float** work,
                     float** DI, int2** tn, int** ln, int2** tm, int** lm, float** partial,
-                    double** trb) {
+                    double** trb, __nv_bfloat16** Vw) {
     *st = c.take<DevStatus>(1);
     *recs = c.take<IterRecord>(iters + 2);
     const bool xcopy = (dtype == FFH_F32 && tc) || (dtype == FFH_BF16 && !x_dev);
@@ -422,10 +433,11 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
     *partial = tc ? c.take<float>(std::max(gram_partial_bytes(pn), gram_partial_bytes(pm)) / 4)
                   : nullptr;
     *trb = c.take<double>(8);
+    *Vw = tc ? c.take<__nv_bfloat16>((size_t)N * pad8(D)) : nullptr;
   };
   DevStatus* st;
   IterRecord* recs;
-  __nv_bfloat16 *Xb, *Gb, *Mb;
+  __nv_bfloat16 *Xb, *Gb, *Mb, *Vw;
   float *stage, *q, *r, *A2, *B2, *L, *Linv, *work, *DI, *partial;
   int2 *tn, *tm;
   int *ln, *lm;
@@ -433,13 +445,13 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
   {
     Carve c(nullptr);
     layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &DI, &tn,
-           &ln, &tm, &lm, &partial, &trb);
+           &ln, &tm, &lm, &partial, &trb, &Vw);
     ffh_status es = ensure_ws(h, c.off + 1024);
     if (es) return es;
   }
   Carve c(h->ws);
   layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &DI, &tn, &ln,
-         &tm, &lm, &partial, &trb);
+         &tm, &lm, &partial, &trb, &Vw);
   cudaStream_t s = h->stream;
   CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
   CK(cudaMemsetAsync(recs, 0, sizeof(IterRecord) * (iters + 2), s));
@@ -515,7 +527,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
       if (t > 1) CK(launch_dot(q, r, N, &recs[t - 1].sum_qr_A, s));
     }
     // ---- B-update
-    es = gram(h, gs, N, m, q, sB, B[nxt], partial, gtm, st);
+    es = gram(h, gs, N, m, q, sB, B[nxt], partial, gtm, st, Vw);
     if (es) return es;
     if (frob) {
       CK(launch_frob2(A[cur], n, trb + 4, s));
@@ -534,7 +546,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
     if (es) return es;
     CK(launch_dot(q, r, N, &R->sum_qr_B, s));
     // ---- A-update
-    es = gram(h, xs, N, n, r, sA, A[nxt], partial, gtn, st);
+    es = gram(h, xs, N, n, r, sA, A[nxt], partial, gtn, st, Vw);
     if (es) return es;
     if (frob) {
       CK(launch_frob2(B[nxt], m, trb + 5, s));

@@ -104,7 +104,8 @@ struct GramArgs {
 };
 
 __global__ void __launch_bounds__(gram::THREADS, 1)
-    k_gram_tc(const __grid_constant__ CUtensorMap tmap, const GramArgs a) {
+    k_gram_tc(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
+              const GramArgs a) {
   using namespace gram;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -142,7 +143,10 @@ __global__ void __launch_bounds__(gram::THREADS, 1)
     tmem_alloc(tmem_slot, TMEM_COLS);
     tmem_relinquish();
   }
-  if (warp == 0 && lane == 0) prefetch_tmap(&tmap);
+  if (warp == 0 && lane == 0) {
+    prefetch_tmap(&amap);
+    prefetch_tmap(&bmap);
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -174,10 +178,10 @@ __global__ void __launch_bounds__(gram::THREADS, 1)
             const int y = kb * BK;
 #pragma unroll
             for (int c = 0; c < BM / 64; ++c)
-              tma_load_2d(sa + c * BOX_BYTES, &tmap, &full[s], tt.x * BM + c * 64, y);
+              tma_load_2d(sa + c * BOX_BYTES, &amap, &full[s], tt.x * BM + c * 64, y);
 #pragma unroll
             for (int c = 0; c < BN / 64; ++c)
-              tma_load_2d(sb + c * BOX_BYTES, &tmap, &full[s], tt.y * BN + c * 64, y);
+              tma_load_2d(sb + c * BOX_BYTES, &bmap, &full[s], tt.y * BN + c * 64, y);
             if (a.w) bulk_load(wbuf + s * BK, a.w + (size_t)kb * BK, BK * 4, &full[s]);
           }
         }
@@ -406,10 +410,17 @@ size_t gram_partial_bytes(const GramPlan& p) {
 cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t ld,
                            const float* w_padded, float scale, float* C, int64_t ldc,
                            float* partial, int2* tiles_dev, int* lut_dev, const GramPlan& plan,
-                           DevStatus* st, int fault, cudaStream_t s, cudaEvent_t after_main) {
-  CUtensorMap map;
-  if (!make_map_bf16(&map, V, (uint64_t)d, (uint64_t)N, (uint64_t)ld, 64, gram::BK))
+                           DevStatus* st, int fault, cudaStream_t s, cudaEvent_t after_main,
+                           const __nv_bfloat16* Va, int64_t lda) {
+  CUtensorMap bmap, amap;
+  if (!make_map_bf16(&bmap, V, (uint64_t)d, (uint64_t)N, (uint64_t)ld, 64, gram::BK))
     return cudaErrorInvalidValue;
+  if (Va && w_padded) return cudaErrorInvalidValue;  // a pre-scaled A operand carries the weights
+  if (!Va) {
+    amap = bmap;
+  } else if (!make_map_bf16(&amap, Va, (uint64_t)d, (uint64_t)N, (uint64_t)lda, 64, gram::BK)) {
+    return cudaErrorInvalidValue;
+  }
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(k_gram_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -428,7 +439,7 @@ cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t
   a.st = st;
   a.fault = fault;
   a.budget_ns = fault == FFH_FAULT_LOST_COPY ? kFaultWaitBudgetNs : kWaitBudgetNs;
-  k_gram_tc<<<plan.grid, gram::THREADS, gram::SMEM_BYTES, s>>>(map, a); note_launches(1);
+  k_gram_tc<<<plan.grid, gram::THREADS, gram::SMEM_BYTES, s>>>(amap, bmap, a); note_launches(1);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   if (after_main && (e = cudaEventRecord(after_main, s)) != cudaSuccess) return e;
@@ -436,6 +447,38 @@ cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t
   const int nbn = (int)((d + gram::BN - 1) / gram::BN);
   k_gram_reduce<<<dim3(nb32, nb32), dim3(32, 8), 0, s>>>(partial, lut_dev, nbn, plan.T, plan.S,
                                                          d, scale, C, ldc); note_launches(1);
+  return cudaGetLastError();
+}
+
+// Vw[k][:] = bf16(w_k V[k][:]) (the A operand of an unweighted Gram that equals
+// V^T diag(w) V); rounding as in the in-kernel scaling (fp32 product, one bf16 rounding).
+__global__ void k_scale_rows(const __nv_bfloat16* __restrict__ V, int64_t ld, int64_t N,
+                             int64_t d8, const float* __restrict__ w, __nv_bfloat16* __restrict__ Vw,
+                             int64_t ldw) {
+  const int64_t total = N * d8;
+  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+       idx += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t row = idx / d8, c = idx - row * d8;
+    const float s = w[row];
+    uint4 v = *reinterpret_cast<const uint4*>(V + row * ld + 8 * c);
+    v.x = scale_bf16x2(v.x, s);
+    v.y = scale_bf16x2(v.y, s);
+    v.z = scale_bf16x2(v.z, s);
+    v.w = scale_bf16x2(v.w, s);
+    *reinterpret_cast<uint4*>(Vw + row * ldw + 8 * c) = v;
+  }
+}
+
+cudaError_t launch_scale_rows(const __nv_bfloat16* V, int64_t ld, int64_t N, int64_t d,
+                              const float* w, __nv_bfloat16* Vw, int64_t ldw, cudaStream_t s) {
+  if (d % 8 || ld % 8 || ldw % 8 ||
+      ((reinterpret_cast<uintptr_t>(V) | reinterpret_cast<uintptr_t>(Vw)) & 15))
+    return cudaErrorInvalidValue;
+  const int64_t total = N * (d / 8);
+  if (total == 0) return cudaSuccess;
+  const int64_t blocks = std::min<int64_t>((total + 255) / 256, (int64_t)num_sms() * 8);
+  k_scale_rows<<<(unsigned)blocks, 256, 0, s>>>(V, ld, N, d / 8, w, Vw, ldw);
+  note_launches(1);
   return cudaGetLastError();
 }
 
