@@ -61,7 +61,7 @@ long long launches_so_far();
 // triangle: tile_col * kGramBN <= tile_row * kGramBM + kGramBM - 1
 constexpr int kGramBM = 256;
 constexpr int kGramBN = 256;
-constexpr int kGramBK = 32;   // samples per pipeline stage (weights padded to this)
+constexpr int kGramBK = 64;   // samples per pipeline stage (weights padded to this)
 struct GramPlan {
   int T;        // lower-triangle output tiles
   int S;        // K splits

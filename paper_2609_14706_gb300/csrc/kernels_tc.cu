@@ -81,8 +81,8 @@ __device__ __forceinline__ uint32_t scale_bf16x2(uint32_t v, float s) {
 namespace gram {
 constexpr int BM = kGramBM;  // output rows (features i) per tile: two M = 128 MMAs
 constexpr int BN = kGramBN;  // output cols (features j) per tile
-constexpr int BK = 32;       // samples per pipeline stage
-constexpr int STAGES = 6;
+constexpr int BK = kGramBK;  // samples per pipeline stage
+constexpr int STAGES = 3;    // 3 x 64 KB: fewer, larger stages keep the MMA fed
 constexpr int BOX_BYTES = 64 * BK * 2;  // one TMA box: 64 features x BK samples
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
@@ -216,7 +216,9 @@ __global__ void __launch_bounds__(gram::THREADS, 1)
         for (int kb = kb0; kb < kb1; ++kb, ++it) {
           const int s = it % STAGES;
           const uint32_t ph = (it / STAGES) & 1;
-          if (!mbar_wait(&scaled[s], ph, abort_flag, budget)) {
+          // unweighted: the operands are ready when the TMA lands; weighted: when the
+          // staging warps have scaled A
+          if (!mbar_wait(a.w ? &scaled[s] : &full[s], ph, abort_flag, budget)) {
             ok = false;
             break;
           }
@@ -260,14 +262,14 @@ __global__ void __launch_bounds__(gram::THREADS, 1)
       const int split = u / a.T;
       const int kb0 = static_cast<int>((int64_t)a.KB * split / a.S);
       const int kb1 = static_cast<int>((int64_t)a.KB * (split + 1) / a.S);
-      for (int kb = kb0; kb < kb1; ++kb, ++it) {
+      for (int kb = kb0; kb < kb1 && a.w; ++kb, ++it) {
         const int s = it % STAGES;
         const uint32_t ph = (it / STAGES) & 1;
         if (!mbar_wait(&full[s], ph, abort_flag, a.fault ? kFaultWaitBudgetNs : budget)) {
           ok = false;
           break;
         }
-        if (a.w) {
+        {
           uint4* A4 = reinterpret_cast<uint4*>(stages + s * STAGE_BYTES);
           const float* wr = wbuf + s * BK;
           constexpr int CHUNKS_PER_BOX = BOX_BYTES / 16;
