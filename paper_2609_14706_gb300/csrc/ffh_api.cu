@@ -51,6 +51,7 @@ struct ffh_ctx {
     cudaEvent_t a, b;
   };
   std::vector<Pending> pending;
+  CholStreams chol_cs;  // look-ahead streams of the tensor-core Cholesky (created on first use)
 };
 
 namespace {
@@ -236,6 +237,7 @@ ffh_status ffh_destroy(ffh_t h) {
     cudaFree(h->ws);
   }
   for (cudaEvent_t e : h->ev_pool) cudaEventDestroy(e);
+  chol_streams_destroy(&h->chol_cs);
   delete h;
   return FFH_OK;
 }
@@ -352,10 +354,18 @@ ffh_status qform(ffh_t h, const Staged& V, int64_t N, int64_t d, const float* Li
 ffh_status chol(ffh_t h, const float* F, int64_t d, float* L, float* Linv, float* work, float* DI,
                 DevStatus* st, int fault) {
   cudaEvent_t t0 = prof_begin(h);
-  if (h->opt.kernel == 1)
+  if (h->opt.kernel == 1) {
     CK(launch_cholesky(F, d, d, L, Linv, work, DI, st, fault, h->stream));
-  else
-    CK(launch_cholesky_tc(F, d, d, L, Linv, work, st, fault, h->stream));
+  } else {
+    if (!h->chol_cs.crit) {
+      const cudaError_t e = chol_streams_init(&h->chol_cs);
+      if (e != cudaSuccess) {
+        chol_streams_destroy(&h->chol_cs);
+        return fail(h, FFH_ERR_CUDA, "Cholesky streams: %s", cudaGetErrorString(e));
+      }
+    }
+    CK(launch_cholesky_tc(F, d, d, L, Linv, work, st, fault, h->stream, &h->chol_cs));
+  }
   prof_end(h, PROF_CHOL, t0);
   return FFH_OK;
 }

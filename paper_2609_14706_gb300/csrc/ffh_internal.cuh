@@ -109,9 +109,20 @@ cudaError_t launch_cholesky(const float* F, int64_t d, int64_t ldf, float* L, fl
                             float* work, float* diag_inv, DevStatus* st, int fault,
                             cudaStream_t s);
 size_t cholesky_work_floats(int64_t d);
-// tensor-core Cholesky + inverse (kernels_chol.cu); `work` of cholesky_tc_work_bytes(d)
+// Streams and events of the look-ahead schedule of the tensor-core Cholesky: the panel
+// chain (diagonal block, panel solve, update of the next column block) runs on `crit`
+// (highest priority), the rest of each trailing update on `side` (lowest priority).
+struct CholStreams {
+  cudaStream_t crit = nullptr, side = nullptr;
+  cudaEvent_t ev[5] = {};  // fork, panel solve done, trailing update done (x2), join
+};
+cudaError_t chol_streams_init(CholStreams* cs);
+void chol_streams_destroy(CholStreams* cs);
+// tensor-core Cholesky + inverse (kernels_chol.cu); `work` of cholesky_tc_work_bytes(d).
+// With cs the work forks from s onto cs->crit / cs->side and joins back into s.
 cudaError_t launch_cholesky_tc(const float* F, int64_t d, int64_t ldf, float* L, float* Linv,
-                               void* work, DevStatus* st, int fault, cudaStream_t s);
+                               void* work, DevStatus* st, int fault, cudaStream_t s,
+                               CholStreams* cs = nullptr);
 size_t cholesky_tc_work_bytes(int64_t d);
 cudaError_t launch_fill_identity(float* F, int64_t d, int64_t ld, cudaStream_t s);
 cudaError_t launch_damp(float* F, int64_t d, int64_t ld, float lambda, DevStatus* st,

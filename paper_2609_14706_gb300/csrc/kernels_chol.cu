@@ -622,13 +622,69 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
 size_t cholesky_tc_work_bytes(int64_t d) {
   const int64_t kmax = (d + 63) / 64 * 64;
   const int64_t rows = (d + 127) / 128 * 128 + 128;
-  // W copy, T scratch, four split buffers (each <= rows x 2*kmax bf16)
-  return (size_t)d * d * 4 + (size_t)d * d * 4 + 4 * (size_t)rows * 2 * kmax * 2 + 4096;
+  // W copy, T scratch, five split buffers (each <= rows x 2*kmax bf16)
+  return (size_t)d * d * 4 + (size_t)d * d * 4 + 5 * (size_t)rows * 2 * kmax * 2 + 4096;
 }
 
+cudaError_t chol_streams_init(CholStreams* cs) {
+  int least = 0, greatest = 0;
+  cudaError_t e = cudaDeviceGetStreamPriorityRange(&least, &greatest);
+  if (e != cudaSuccess) return e;
+  if ((e = cudaStreamCreateWithPriority(&cs->crit, cudaStreamNonBlocking, greatest)) != cudaSuccess)
+    return e;
+  if ((e = cudaStreamCreateWithPriority(&cs->side, cudaStreamNonBlocking, least)) != cudaSuccess)
+    return e;
+  for (cudaEvent_t& ev : cs->ev)
+    if ((e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming)) != cudaSuccess) return e;
+  return cudaSuccess;
+}
+
+void chol_streams_destroy(CholStreams* cs) {
+  if (cs->crit) cudaStreamSynchronize(cs->crit);
+  if (cs->side) cudaStreamSynchronize(cs->side);
+  for (cudaEvent_t& ev : cs->ev)
+    if (ev) cudaEventDestroy(ev), ev = nullptr;
+  if (cs->crit) cudaStreamDestroy(cs->crit), cs->crit = nullptr;
+  if (cs->side) cudaStreamDestroy(cs->side), cs->side = nullptr;
+}
+
+static cudaError_t cholesky_tc_body(const float* F, int64_t d, int64_t ldf, float* L, float* Linv,
+                                    void* work, DevStatus* st, int fault, cudaStream_t s,
+                                    CholStreams* cs);
+
 // L (lower), Linv = L^-1 (lower); st->logdet += log|F|.  F is read, not modified.
+// Look-ahead (cs): panel p's trailing update is split into the next column block (on the
+// critical stream, needed by panel p+1) and the columns beyond it (on the side stream,
+// overlapping panel p+1's diagonal block and panel solve).  The update of a column block
+// by panel p-1 (side) finishes before panel p updates the same block (critical), and the
+// panel GEMM output buffer alternates between two splits so that the side stream's reads
+// of panel p's split are not overwritten by panel p+1.
 cudaError_t launch_cholesky_tc(const float* F, int64_t d, int64_t ldf, float* L, float* Linv,
-                               void* work, DevStatus* st, int fault, cudaStream_t s) {
+                               void* work, DevStatus* st, int fault, cudaStream_t s_user,
+                               CholStreams* cs) {
+  cudaError_t e;
+  cudaStream_t s = s_user;
+  if (cs) {
+    if ((e = cudaEventRecord(cs->ev[0], s_user)) != cudaSuccess) return e;
+    if ((e = cudaStreamWaitEvent(cs->crit, cs->ev[0], 0)) != cudaSuccess) return e;
+    if ((e = cudaStreamWaitEvent(cs->side, cs->ev[0], 0)) != cudaSuccess) return e;
+    s = cs->crit;
+  }
+  e = cholesky_tc_body(F, d, ldf, L, Linv, work, st, fault, s, cs);
+  if (cs) {
+    // join: everything on both streams completes before later work on the user stream
+    cudaEventRecord(cs->ev[2], cs->side);
+    cudaStreamWaitEvent(cs->crit, cs->ev[2], 0);
+    cudaEventRecord(cs->ev[4], cs->crit);
+    cudaError_t e2 = cudaStreamWaitEvent(s_user, cs->ev[4], 0);
+    if (e == cudaSuccess) e = e2;
+  }
+  return e;
+}
+
+static cudaError_t cholesky_tc_body(const float* F, int64_t d, int64_t ldf, float* L, float* Linv,
+                                    void* work, DevStatus* st, int fault, cudaStream_t s,
+                                    CholStreams* cs) {
   cudaError_t e;
   const int64_t kmax = (d + 63) / 64 * 64;
   const int64_t rows_cap = (d + 127) / 128 * 128 + 128;
@@ -637,8 +693,8 @@ cudaError_t launch_cholesky_tc(const float* F, int64_t d, int64_t ldf, float* L,
   wp += (size_t)d * d * 4;
   float* T = reinterpret_cast<float*>(wp);
   wp += (size_t)d * d * 4;
-  __nv_bfloat16* sb[4];
-  for (int i = 0; i < 4; ++i) {
+  __nv_bfloat16* sb[5];
+  for (int i = 0; i < 5; ++i) {
     sb[i] = reinterpret_cast<__nv_bfloat16*>(wp);
     wp += (size_t)rows_cap * 2 * kmax * 2;
   }
@@ -670,14 +726,41 @@ cudaError_t launch_cholesky_tc(const float* F, int64_t d, int64_t ldf, float* L,
     if ((e = split(W + (o + LB) * d + o, d, 0, rows, LB, false, a21, s)) != cudaSuccess) return e;
     const int aseg[3] = {0, 0, 128}, bseg[3] = {0, 128, 0};
     // the epilogue also writes the split of L21 for the trailing update
-    Split l21{sb[2], (int)((rows + 127) / 128 * 128), 128, 1};
+    const int rows_pad = (rows + 127) / 128 * 128;
+    Split l21{sb[cs ? 2 + 2 * (p & 1) : 2], rows_pad, 128, 1};
     if ((e = gemm_tc(a21, m11, 3, aseg, bseg, 128, L + (o + LB) * d + o, d, 0, rows, LB, 1.f,
                      0.f, false, 1, st, s, &l21)) != cudaSuccess)
       return e;
-    // A22 -= L21 L21^T (lower tiles)
-    if ((e = gemm_tc(l21, l21, 3, aseg, bseg, 128, W + (o + LB) * d + (o + LB), d, 0, rows, rows,
-                     -1.f, 1.f, true, 1, st, s)) != cudaSuccess)
+    if (!cs) {
+      // A22 -= L21 L21^T (lower tiles)
+      if ((e = gemm_tc(l21, l21, 3, aseg, bseg, 128, W + (o + LB) * d + (o + LB), d, 0, rows,
+                       rows, -1.f, 1.f, true, 1, st, s)) != cudaSuccess)
+        return e;
+      continue;
+    }
+    // side: columns beyond the next block, A22[128:, 128:] -= L21[128:] L21[128:]^T
+    if ((e = cudaEventRecord(cs->ev[1], s)) != cudaSuccess) return e;
+    if ((e = cudaStreamWaitEvent(cs->side, cs->ev[1], 0)) != cudaSuccess) return e;
+    if (rows > LB) {
+      Split rest{l21.p + (size_t)LB * 2 * l21.kpad, rows_pad - LB, 128, 1};
+      if ((e = gemm_tc(rest, rest, 3, aseg, bseg, 128, W + (o + 2 * LB) * d + (o + 2 * LB), d, 0,
+                       rows - LB, rows - LB, -1.f, 1.f, true, 1, st, cs->side)) != cudaSuccess)
+        return e;
+    }
+    if ((e = cudaEventRecord(cs->ev[2 + (p & 1)], cs->side)) != cudaSuccess) return e;
+    // critical: the next column block, A22[:, :128] -= L21 L21[:128]^T, after the side
+    // stream's update of the same block by the previous panel
+    if (p > 0 && (e = cudaStreamWaitEvent(s, cs->ev[2 + ((p - 1) & 1)], 0)) != cudaSuccess)
       return e;
+    Split head{l21.p, LB, 128, 1};
+    if ((e = gemm_tc(l21, head, 3, aseg, bseg, 128, W + (o + LB) * d + (o + LB), d, 0, rows,
+                     rows < LB ? rows : LB, -1.f, 1.f, true, 1, st, s)) != cudaSuccess)
+      return e;
+  }
+  if (cs) {
+    // the side stream's last updates precede the inverse
+    if ((e = cudaEventRecord(cs->ev[2 + (np & 1)], cs->side)) != cudaSuccess) return e;
+    if ((e = cudaStreamWaitEvent(s, cs->ev[2 + (np & 1)], 0)) != cudaSuccess) return e;
   }
   if (!Linv) return cudaSuccess;
   // inverse by recursive doubling over block size b = 128, 256, ...
