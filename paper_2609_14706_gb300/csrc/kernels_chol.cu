@@ -27,6 +27,31 @@ using namespace ptx;
 
 static constexpr uint64_t kGemmWaitNs = 4000000000ull;
 
+// Programmatic dependent launch: the kernels of the panel chain start (launch, CTA
+// placement) while their predecessor in the stream is still running, and wait for it to
+// finish, with its memory visible, before touching any data (griddepcontrol.wait).  A
+// kernel lets its dependent start as soon as all of its own CTAs are resident.
+__device__ __forceinline__ void pdl_enter() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+static cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 static PFN_cuTensorMapEncodeTiled_v12000 encode_fn_chol() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
   if (!fn) {
@@ -87,6 +112,7 @@ __global__ void __launch_bounds__(256, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
               const GemmTcArgs a) {
   using namespace gt;
+  pdl_enter();
   const int tn = blockIdx.x, tm = blockIdx.y, z = blockIdx.z;
   const int row0 = tm * BM, col0 = tn * BN;
   if (a.lower_only && col0 > row0 + BM - 1) return;
@@ -284,9 +310,9 @@ static cudaError_t gemm_tc(const Split& A, const Split& B, int nseg, const int a
   g.split_rows_pad = out_split ? out_split->rows_pad : 0;
   g.st = st;
   dim3 grid((N + gt::BN - 1) / gt::BN, (M + gt::BM - 1) / gt::BM, batch);
-  k_gemm_tc<<<grid, 256, gt::SMEM_BYTES, s>>>(am, bm, g);
+  cudaError_t e = launch_pdl(k_gemm_tc, grid, dim3(256), gt::SMEM_BYTES, s, am, bm, g);
   note_launches(1);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 // ---------------------------------------------------------------------------
@@ -300,6 +326,7 @@ static cudaError_t gemm_tc(const Split& A, const Split& B, int nseg, const int a
 __global__ void k_split_hilo(const float* __restrict__ src, int64_t lds, int64_t src_stride,
                              int rows, int cols, int trans, __nv_bfloat16* __restrict__ dst,
                              int rows_pad, int kpad, int batch) {
+  pdl_enter();
   const int64_t per = (int64_t)rows_pad * kpad;
   const int64_t total = per * batch;
   for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
@@ -325,10 +352,11 @@ static cudaError_t split(const float* src, int64_t lds, int64_t src_stride, int 
   const int64_t total = (int64_t)d.rows_pad * d.kpad * d.batch;
   if (total == 0) return cudaSuccess;
   const int64_t blocks = std::min<int64_t>((total + 255) / 256, (int64_t)num_sms() * 16);
-  k_split_hilo<<<(unsigned)blocks, 256, 0, s>>>(src, lds, src_stride, rows, cols, trans ? 1 : 0,
-                                                d.p, d.rows_pad, d.kpad, d.batch);
+  cudaError_t e = launch_pdl(k_split_hilo, dim3((unsigned)blocks), dim3(256), 0, s, src, lds,
+                             src_stride, rows, cols, trans ? 1 : 0, d.p, d.rows_pad, d.kpad,
+                             d.batch);
   note_launches(1);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 // ---------------------------------------------------------------------------
@@ -484,6 +512,7 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
   float* Ptb = Ms + LB * LP;           // [2][32][PTP] transposed sub-panels
   float* Mtb = Ptb + 2 * 32 * PTP;     // [2][32][MTP] transposed diagonal-block inverses
   float* T = Mtb + 2 * 32 * MTP;       // [32][TP]
+  pdl_enter();
   const int b = (int)((d - o) < LB ? (d - o) : LB);
   const int tid = threadIdx.x, warp = tid >> 5;
   for (int idx = tid; idx < LB * LB / 4; idx += LEAF_THREADS) {
@@ -715,15 +744,21 @@ static cudaError_t cholesky_tc_body(const float* F, int64_t d, int64_t ldf, floa
   const int np = (int)((d + LB - 1) / LB);
   for (int p = 0; p < np; ++p) {
     const int64_t o = (int64_t)p * LB;
-    k_chol_leaf<<<1, LEAF_THREADS, LB_SMEM, s>>>(W, d, d, o, L, d, Mdiag, d, sb[1], st, fault);
+    if ((e = launch_pdl(k_chol_leaf, dim3(1), dim3(LEAF_THREADS), LB_SMEM, s, W, d, d, o, L, d,
+                        Mdiag, d, sb[1], st, fault)) != cudaSuccess)
+      return e;
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     const int rows = (int)(d - o - LB);
     if (rows <= 0) continue;
-    // L21 = A21 * M11^T : A' = split(A21) (rows x 128), B' = split(M11) (128 x 128)
-    Split a21{sb[0], (int)((rows + 127) / 128 * 128), 128, 1};
+    // L21 = A21 * M11^T : A' = split(A21) (rows x 128), B' = split(M11) (128 x 128).  The
+    // A21 split sits 128 rows into sb[0]: with look-ahead the previous panel's update of
+    // this column block writes it from its epilogue (rows of the diagonal block first).
+    Split a21{sb[0] + (size_t)LB * 2 * 128, (int)((rows + 127) / 128 * 128), 128, 1};
     Split m11{sb[1], 128, 128, 1};
-    if ((e = split(W + (o + LB) * d + o, d, 0, rows, LB, false, a21, s)) != cudaSuccess) return e;
+    if ((!cs || p == 0) &&
+        (e = split(W + (o + LB) * d + o, d, 0, rows, LB, false, a21, s)) != cudaSuccess)
+      return e;
     const int aseg[3] = {0, 0, 128}, bseg[3] = {0, 128, 0};
     // the epilogue also writes the split of L21 for the trailing update
     const int rows_pad = (rows + 127) / 128 * 128;
@@ -753,8 +788,10 @@ static cudaError_t cholesky_tc_body(const float* F, int64_t d, int64_t ldf, floa
     if (p > 0 && (e = cudaStreamWaitEvent(s, cs->ev[2 + ((p - 1) & 1)], 0)) != cudaSuccess)
       return e;
     Split head{l21.p, LB, 128, 1};
+    Split next_a21{sb[0], rows_pad + LB, 128, 1};  // the next panel's A21 split (see above)
     if ((e = gemm_tc(l21, head, 3, aseg, bseg, 128, W + (o + LB) * d + (o + LB), d, 0, rows,
-                     rows < LB ? rows : LB, -1.f, 1.f, true, 1, st, s)) != cudaSuccess)
+                     rows < LB ? rows : LB, -1.f, 1.f, true, 1, st, s,
+                     rows > LB ? &next_a21 : nullptr)) != cudaSuccess)
       return e;
   }
   if (cs) {
