@@ -384,13 +384,17 @@ constexpr int PTP = LB + 4;  // pitch of Pt (float4 rows)
 constexpr int MTP = 36;      // pitch of Mt
 constexpr int TP = 100;      // pitch of the 32 x 96 scratch T
 constexpr int LB_SMEM =
-    (2 * LB * LP + 2 * 32 * PTP + 2 * 32 * MTP + 32 * TP) * 4 + 64;
+    (2 * LB * LP + 2 * 32 * PTP + 2 * 32 * MTP + 32 * TP + LB + 64) * 4 + 64;
 constexpr int LEAF_THREADS = 512;
 
-// A(q): factor and invert the diagonal block (warp 0 only).  Returns sum log(pivot)
-// (fp32: FP64 arithmetic is slow on this part and would sit on the pivot chain).
-__device__ __forceinline__ float leaf_diag(float* Ls, float* Ms, float* Mt, int c0,
-                                            int64_t o, DevStatus* st, bool& bad) {
+// A(q): factor and invert the diagonal block (warp 0 only); the pivots go to pivs[c0..].
+// The column of l values of pivot j reaches the other lanes through a shared buffer
+// written rotated (slot (lane - j - 1) mod 32 holds lane lane's value), so the 31 values
+// l_{j+1..j+31, j} are eight broadcast float4 loads; the buffer alternates by the parity of
+// j, so one warp barrier per pivot suffices.
+__device__ __forceinline__ void leaf_diag(float* Ls, float* Ms, float* Mt, float* lbuf,
+                                          float* pivs, int c0, int64_t o, DevStatus* st,
+                                          bool& bad) {
   const int lane = threadIdx.x & 31;
   constexpr unsigned FULL = 0xffffffffu;
   float a[32], mc[32];
@@ -399,7 +403,6 @@ __device__ __forceinline__ float leaf_diag(float* Ls, float* Ms, float* Mt, int 
     a[k] = (k <= lane) ? Ls[(c0 + lane) * LP + c0 + k] : 0.f;
     mc[k] = (k == lane) ? 1.f : 0.f;
   }
-  float lg = 0.f;
 #pragma unroll 1
   for (int j = 0; j < 32; ++j) {
     // registers k = 0..31 hold columns j+k of row `lane` (of D) and rows j+k of column
@@ -414,21 +417,31 @@ __device__ __forceinline__ float leaf_diag(float* Ls, float* Ms, float* Mt, int 
     const float r = rsqrtf(piv);
     const float l = a[0] * r;   // lane > j: l_{lane,j}; lane j: sqrt(pivot)
     const float m = mc[0] * r;  // Mi[j][lane] (exactly 0 for lane > j)
-    lg += logf(piv);
+    float* lb = lbuf + (j & 1) * 32;
+    lb[(lane - j - 1) & 31] = l;
+    if (lane == 0) pivs[c0 + j] = piv;
     Ls[(c0 + lane) * LP + c0 + j] = lane >= j ? l : 0.f;
     Ms[(c0 + j) * LP + c0 + lane] = m;
     Mt[lane * MTP + j] = m;
+    __syncwarp();
+    float lk[32];
+#pragma unroll
+    for (int k4 = 0; k4 < 8; ++k4) {
+      const float4 v = *reinterpret_cast<const float4*>(lb + 4 * k4);
+      lk[4 * k4] = v.x;
+      lk[4 * k4 + 1] = v.y;
+      lk[4 * k4 + 2] = v.z;
+      lk[4 * k4 + 3] = v.w;
+    }
 #pragma unroll
     for (int k = 1; k < 32; ++k) {
-      // l_{j+k, j}; for j + k > 31 the value is unused (shifted past the block)
-      const float lk = __shfl_sync(FULL, l, (j + k) & 31);
-      a[k - 1] = fmaf(-l, lk, a[k]);
-      mc[k - 1] = fmaf(-lk, m, mc[k]);
+      // lk[k-1] = l_{j+k, j}; for j + k > 31 the value is unused (shifted past the block)
+      a[k - 1] = fmaf(-l, lk[k - 1], a[k]);
+      mc[k - 1] = fmaf(-lk[k - 1], m, mc[k]);
     }
     a[31] = 0.f;
     mc[31] = 0.f;
   }
-  return lg;
 }
 
 // Rank-32 update of one 4 x 4 block of the trailing lower triangle from the transposed
@@ -512,9 +525,11 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
   float* Ptb = Ms + LB * LP;           // [2][32][PTP] transposed sub-panels
   float* Mtb = Ptb + 2 * 32 * PTP;     // [2][32][MTP] transposed diagonal-block inverses
   float* T = Mtb + 2 * 32 * MTP;       // [32][TP]
+  float* pivs = T + 32 * TP;           // [LB] pivots
+  float* lbuf = pivs + LB;             // [2][32] pivot-column broadcast (warp 0)
   pdl_enter();
   const int b = (int)((d - o) < LB ? (d - o) : LB);
-  const int tid = threadIdx.x, warp = tid >> 5;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   for (int idx = tid; idx < LB * LB / 4; idx += LEAF_THREADS) {
     const int i = idx >> 5, j4 = (idx & 31) * 4;
     float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -543,8 +558,7 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
   if (tid == 0 && fault == FFH_FAULT_BAD_PIVOT && o == 0) Ls[0] = __int_as_float(0x7fc00000);
   __syncthreads();
   bool bad = false;
-  float lg = 0.f;  // held by warp 0
-  if (warp == 0) lg += leaf_diag(Ls, Ms, Mtb, 0, o, st, bad);
+  if (warp == 0) leaf_diag(Ls, Ms, Mtb, lbuf, pivs, 0, o, st, bad);
   __syncthreads();
 #pragma unroll 1
   for (int q = 0; q < 4; ++q) {
@@ -591,7 +605,7 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
         if (bj <= bi) leaf_trail_block(Ls, Pt, c0 + 32 + 4 * bi, c0 + 32 + 4 * bj);
         asm volatile("bar.sync 1, 64;" ::: "memory");
         if (warp == 0)
-          lg += leaf_diag(Ls, Ms, Mtb + ((q + 1) & 1) * 32 * MTP, c0 + 32, o, st, bad);
+          leaf_diag(Ls, Ms, Mtb + ((q + 1) & 1) * 32 * MTP, lbuf, pivs, c0 + 32, o, st, bad);
       } else {
         const int t = tid - 64;
         for (int blk = t; blk < nb * nb; blk += LEAF_THREADS - 64) {
@@ -645,7 +659,13 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
       *reinterpret_cast<uint2*>(m11_split + i * 2 * LB + LB + j0) = *reinterpret_cast<uint2*>(lo);
     }
   }
-  if (tid == 0) atomicAdd(&st->logdet, (double)lg);
+  if (warp == 0) {
+    // log|F11| = sum_j log(pivot_j), off the pivot chain
+    float lg = 0.f;
+    for (int i = lane; i < LB; i += 32) lg += logf(pivs[i]);
+    for (int off = 16; off > 0; off >>= 1) lg += __shfl_down_sync(0xffffffffu, lg, off);
+    if (lane == 0) atomicAdd(&st->logdet, (double)lg);
+  }
 }
 
 size_t cholesky_tc_work_bytes(int64_t d) {
