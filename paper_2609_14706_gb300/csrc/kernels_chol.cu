@@ -391,8 +391,9 @@ constexpr int LEAF_THREADS = 512;
 // The column of l values of pivot j reaches the other lanes through a shared buffer
 // written rotated (slot (lane - j - 1) mod 32 holds lane lane's value), so the 31 values
 // l_{j+1..j+31, j} are eight broadcast float4 loads; the buffer alternates by the parity of
-// j, so one warp barrier per pivot suffices.
-__device__ __forceinline__ void leaf_diag(float* Ls, float* Ms, float* Mt, float* lbuf,
+// j, so one warp barrier per pivot suffices.  Not inlined: one copy serves the four
+// sub-panels (measured faster than the inlined copies).
+__device__ __noinline__ void leaf_diag(float* Ls, float* Ms, float* Mt, float* lbuf,
                                           float* pivs, int c0, int64_t o, DevStatus* st,
                                           bool& bad) {
   const int lane = threadIdx.x & 31;
