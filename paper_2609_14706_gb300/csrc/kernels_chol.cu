@@ -372,7 +372,8 @@ static cudaError_t split(const float* src, int64_t lds, int64_t src_stride, int 
 //   C(q)  warps 0-1 apply the rank-32 update of sub-panel q to D_{q+1} and warp 0 goes
 //         on to A(q+1), while warps 2-15 update the rest of the trailing lower triangle
 //         and form row block q of the inverse by block forward substitution,
-//         M[Q][0:32q] = -Mi_q (L[Q][0:32q] M[0:32q][0:32q]).
+//         M[Q][0:32q] = -Mi_q T_q, and the product T_{q+1} = L[Q+1][0:32q+32] M[..][..]
+//         of the next row block (only -Mi_3 T_3 is left after the last sub-panel).
 // Pt and Mt are double-buffered by the parity of q, so A(q+1) never writes what C(q)
 // reads.  The pivot product gives log|F11| = sum_j log(pivot_j).
 // Outputs: L11 and M11 (fp32) and the bf16 hi/lo split of M11 ([hi | lo] rows, pitch
@@ -381,10 +382,11 @@ static cudaError_t split(const float* src, int64_t lds, int64_t src_stride, int 
 constexpr int LB = 128;
 constexpr int LP = LB + 1;   // pitch of the row-major 128 x 128 blocks (conflict-free columns)
 constexpr int PTP = LB + 4;  // pitch of Pt (float4 rows)
+constexpr int MP = LB + 4;   // pitch of M11 (float4 rows)
 constexpr int MTP = 36;      // pitch of Mt
 constexpr int TP = 100;      // pitch of the 32 x 96 scratch T
 constexpr int LB_SMEM =
-    (2 * LB * LP + 2 * 32 * PTP + 2 * 32 * MTP + 32 * TP + LB + 64) * 4 + 64;
+    (LB * LP + LB * MP + 2 * 32 * PTP + 2 * 32 * MTP + 32 * TP + LB + 64) * 4 + 64;
 constexpr int LEAF_THREADS = 512;
 
 // A(q): factor and invert the diagonal block (warp 0 only); the pivots go to pivs[c0..].
@@ -422,7 +424,7 @@ __device__ __noinline__ void leaf_diag(float* Ls, float* Ms, float* Mt, float* l
     lb[(lane - j - 1) & 31] = l;
     if (lane == 0) pivs[c0 + j] = piv;
     Ls[(c0 + lane) * LP + c0 + j] = lane >= j ? l : 0.f;
-    Ms[(c0 + j) * LP + c0 + lane] = m;
+    Ms[(c0 + j) * MP + c0 + lane] = m;
     Mt[lane * MTP + j] = m;
     __syncwarp();
     float lk[32];
@@ -466,52 +468,58 @@ __device__ __forceinline__ void leaf_trail_block(float* Ls, const float* Pt, int
       if (cc0 + jx <= r0 + i) Ls[(r0 + i) * LP + cc0 + jx] -= acc[i][jx];
 }
 
-// Row block q >= 1 of the inverse: T = L[Q][0:c0] M[0:c0][0:c0], then
-// M[Q][0:c0] = -Mi_q T.  Threads t = 0..nt-1; `sync` separates the two products.
-template <class Sync>
-__device__ __forceinline__ void leaf_inverse_rows(float* Ls, float* Ms, float* T, int c0, int t,
-                                                  int nt, Sync sync) {
+// Row block Q = [c0, c0 + 32) (c0 >= 32) of the inverse, left of the diagonal block, in
+// two products: T = L[Q][0:c0] M[0:c0][0:c0] (needs the rows of M above Q), then
+// M[Q][0:c0] = -Mi_Q T (needs the diagonal block's inverse Mi_Q).  Threads t = 0..nt-1.
+__device__ __forceinline__ void leaf_inverse_T(const float* Ls, const float* Ms, float* T, int c0,
+                                               int t, int nt) {
   const int nbx = c0 / 4;  // 4-wide column blocks of [0, c0)
-  for (int blk = t; blk < 8 * nbx; blk += nt) {
-    const int i0 = (blk / nbx) * 4, x0 = (blk % nbx) * 4;
-    float acc[4][4] = {};
+  // 2 rows x 4 columns per thread
+  for (int blk = t; blk < 16 * nbx; blk += nt) {
+    const int i0 = (blk / nbx) * 2, x0 = (blk % nbx) * 4;
+    float acc[2][4] = {};
     // M lower triangular: M[k][x] = 0 for k < x, so k starts at x0
     for (int k = x0; k < c0; ++k) {
-      float av[4], bv[4];
+      float av[2];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) av[i] = Ls[(c0 + i0 + i) * LP + k];
-#pragma unroll
-      for (int jx = 0; jx < 4; ++jx) bv[jx] = Ms[k * LP + x0 + jx];
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int jx = 0; jx < 4; ++jx) acc[i][jx] = fmaf(av[i], bv[jx], acc[i][jx]);
-    }
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-      *reinterpret_cast<float4*>(T + (i0 + i) * TP + x0) =
-          make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
-  }
-  sync();
-  for (int blk = t; blk < 8 * nbx; blk += nt) {
-    const int i0 = (blk / nbx) * 4, x0 = (blk % nbx) * 4;
-    float acc[4][4] = {};
-    // Mi_q lower triangular: row i needs j <= i < i0 + 4
-    for (int j = 0; j < i0 + 4; ++j) {
-      float av[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) av[i] = Ms[(c0 + i0 + i) * LP + c0 + j];
-      const float4 bv = *reinterpret_cast<const float4*>(T + j * TP + x0);
+      for (int i = 0; i < 2; ++i) av[i] = Ls[(c0 + i0 + i) * LP + k];
+      const float4 bv = *reinterpret_cast<const float4*>(Ms + k * MP + x0);
       const float br[4] = {bv.x, bv.y, bv.z, bv.w};
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
+      for (int i = 0; i < 2; ++i)
 #pragma unroll
         for (int jx = 0; jx < 4; ++jx) acc[i][jx] = fmaf(av[i], br[jx], acc[i][jx]);
     }
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
+    for (int i = 0; i < 2; ++i)
+      *reinterpret_cast<float4*>(T + (i0 + i) * TP + x0) =
+          make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+  }
+}
+
+__device__ __forceinline__ void leaf_inverse_apply(float* Ms, const float* T, int c0, int t,
+                                                   int nt) {
+  const int nbx = c0 / 4;
+  // 2 rows x 4 columns per thread
+  for (int blk = t; blk < 16 * nbx; blk += nt) {
+    const int i0 = (blk / nbx) * 2, x0 = (blk % nbx) * 4;
+    float acc[2][4] = {};
+    // Mi lower triangular: row i needs j <= i < i0 + 2
+    for (int j = 0; j < i0 + 2; ++j) {
+      float av[2];
 #pragma unroll
-      for (int jx = 0; jx < 4; ++jx) Ms[(c0 + i0 + i) * LP + x0 + jx] = -acc[i][jx];
+      for (int i = 0; i < 2; ++i) av[i] = Ms[(c0 + i0 + i) * MP + c0 + j];
+      const float4 bv = *reinterpret_cast<const float4*>(T + j * TP + x0);
+      const float br[4] = {bv.x, bv.y, bv.z, bv.w};
+#pragma unroll
+      for (int i = 0; i < 2; ++i)
+#pragma unroll
+        for (int jx = 0; jx < 4; ++jx) acc[i][jx] = fmaf(av[i], br[jx], acc[i][jx]);
+    }
+#pragma unroll
+    for (int i = 0; i < 2; ++i)
+#pragma unroll
+      for (int jx = 0; jx < 4; ++jx) Ms[(c0 + i0 + i) * MP + x0 + jx] = -acc[i][jx];
   }
 }
 
@@ -522,8 +530,8 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
                                                                DevStatus* st, int fault) {
   extern __shared__ float sh[];
   float* Ls = sh;                      // [LB][LP]  working block -> L11
-  float* Ms = Ls + LB * LP;            // [LB][LP]  M11
-  float* Ptb = Ms + LB * LP;           // [2][32][PTP] transposed sub-panels
+  float* Ms = Ls + LB * LP;            // [LB][MP]  M11
+  float* Ptb = Ms + LB * MP;           // [2][32][PTP] transposed sub-panels
   float* Mtb = Ptb + 2 * 32 * PTP;     // [2][32][MTP] transposed diagonal-block inverses
   float* T = Mtb + 2 * 32 * MTP;       // [32][TP]
   float* pivs = T + 32 * TP;           // [LB] pivots
@@ -552,7 +560,7 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
       float x = (j <= i) ? vv[e] : 0.f;
       if (i >= b || j >= b) x = (i == j) ? 1.f : 0.f;  // identity padding
       Ls[i * LP + j] = x;
-      Ms[i * LP + j] = 0.f;
+      Ms[i * MP + j] = 0.f;
     }
   }
   __syncthreads();
@@ -614,12 +622,15 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
           if (bi < 8 || bj > bi) continue;
           leaf_trail_block(Ls, Pt, c0 + 32 + 4 * bi, c0 + 32 + 4 * bj);
         }
-        if (q >= 1)
-          leaf_inverse_rows(Ls, Ms, T, c0, t, LEAF_THREADS - 64,
-                            [] { asm volatile("bar.sync 2, 448;" ::: "memory"); });
+        // row block q of the inverse (T_q from the previous sub-panel), then T_{q+1}
+        if (q >= 1) {
+          leaf_inverse_apply(Ms, T, c0, t, LEAF_THREADS - 64);
+          asm volatile("bar.sync 2, 448;" ::: "memory");
+        }
+        leaf_inverse_T(Ls, Ms, T, c0 + 32, t, LEAF_THREADS - 64);
       }
     } else {
-      leaf_inverse_rows(Ls, Ms, T, c0, tid, LEAF_THREADS, [] { __syncthreads(); });
+      leaf_inverse_apply(Ms, T, c0, tid, LEAF_THREADS);
     }
     __syncthreads();
   }
@@ -633,7 +644,7 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
     for (int e = 0; e < 4; ++e) {
       const int j = j0 + e;
       lv[e] = (j <= i) ? Ls[i * LP + j] : 0.f;
-      mv[e] = (j <= i && i < b && j < b) ? Ms[i * LP + j] : 0.f;
+      mv[e] = (j <= i && i < b && j < b) ? Ms[i * MP + j] : 0.f;
     }
     if (i < b) {
       if (vec_ok && j0 + 3 < b) {
