@@ -370,7 +370,8 @@ static cudaError_t split(const float* src, int64_t lds, int64_t src_stride, int 
 //   B(q)  all warps: the rows below, L[r][Q] = A[r][Q] Mi_q^T (4 x 4 register blocks),
 //         also stored transposed, Pt[k][r] = L[r][32q+k].
 //   C(q)  warps 0-1 apply the rank-32 update of sub-panel q to D_{q+1} and warp 0 goes
-//         on to A(q+1), while warps 2-15 update the rest of the trailing lower triangle
+//         on to A(q+1), while 11 other warps (not 4, 8, 12, which share warp 0's
+//         scheduler partition) update the rest of the trailing lower triangle
 //         and form row block q of the inverse by block forward substitution,
 //         M[Q][0:32q] = -Mi_q T_q, and the product T_{q+1} = L[Q+1][0:32q+32] M[..][..]
 //         of the next row block (only -Mi_3 T_3 is left after the last sub-panel).
@@ -615,19 +616,22 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
         asm volatile("bar.sync 1, 64;" ::: "memory");
         if (warp == 0)
           leaf_diag(Ls, Ms, Mtb + ((q + 1) & 1) * 32 * MTP, lbuf, pivs, c0 + 32, o, st, bad);
-      } else {
-        const int t = tid - 64;
-        for (int blk = t; blk < nb * nb; blk += LEAF_THREADS - 64) {
+      } else if (warp & 3) {
+        // warps 2, 3, 5-7, 9-11, 13-15: warps 4, 8 and 12 stay idle so that warp 0's
+        // pivot chain has its scheduler partition to itself
+        constexpr int NT = 11 * 32;
+        const int t = (warp - 2 - (warp >> 2)) * 32 + (tid & 31);
+        for (int blk = t; blk < nb * nb; blk += NT) {
           const int bi = blk / nb, bj = blk - (blk / nb) * nb;
           if (bi < 8 || bj > bi) continue;
           leaf_trail_block(Ls, Pt, c0 + 32 + 4 * bi, c0 + 32 + 4 * bj);
         }
         // row block q of the inverse (T_q from the previous sub-panel), then T_{q+1}
         if (q >= 1) {
-          leaf_inverse_apply(Ms, T, c0, t, LEAF_THREADS - 64);
-          asm volatile("bar.sync 2, 448;" ::: "memory");
+          leaf_inverse_apply(Ms, T, c0, t, NT);
+          asm volatile("bar.sync 2, 352;" ::: "memory");
         }
-        leaf_inverse_T(Ls, Ms, T, c0 + 32, t, LEAF_THREADS - 64);
+        leaf_inverse_T(Ls, Ms, T, c0 + 32, t, NT);
       }
     } else {
       leaf_inverse_apply(Ms, T, c0, tid, LEAF_THREADS);
