@@ -548,20 +548,38 @@ cudaError_t launch_normalize(float* A, int64_t n, float* B, int64_t m, IterRecor
   return cudaGetLastError();
 }
 
-// sum (F/trF - P/trP)^2 and sum (F/trF)^2 (trF, trP read from device doubles)
+// sum (F/trF - P/trP)^2 and sum (F/trF)^2 (trF, trP read from device doubles).  Per
+// element in fp32, float4 loads, per-thread partial sums (a few dozen terms) in fp32 and
+// the block and grid sums in fp64: FP64 arithmetic per element is slow on this part, and
+// the statistic needs only a few significant digits.
 __global__ void k_delta(const float* F, const float* P, int64_t total, const double* trF,
                         const double* trP, double* d2, double* n2) {
-  const double a = 1.0 / *trF, b = 1.0 / *trP;
-  double sd = 0.0, sn = 0.0;
-  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
-       idx += (int64_t)gridDim.x * blockDim.x) {
-    const double f = F[idx] * a, p = P[idx] * b;
-    sd += (f - p) * (f - p);
-    sn += f * f;
+  const float a = (float)(1.0 / *trF), b = (float)(1.0 / *trP);
+  float sdf = 0.f, snf = 0.f;
+  const int64_t t0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const bool vec = ((reinterpret_cast<uintptr_t>(F) | reinterpret_cast<uintptr_t>(P)) & 15) == 0;
+  const int64_t n4 = vec ? total / 4 : 0;
+  for (int64_t i = t0; i < n4; i += stride) {
+    const float4 fv = reinterpret_cast<const float4*>(F)[i];
+    const float4 pv = reinterpret_cast<const float4*>(P)[i];
+    const float f[4] = {fv.x * a, fv.y * a, fv.z * a, fv.w * a};
+    const float p[4] = {pv.x * b, pv.y * b, pv.z * b, pv.w * b};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float dd = f[e] - p[e];
+      sdf = fmaf(dd, dd, sdf);
+      snf = fmaf(f[e], f[e], snf);
+    }
   }
-  sd = block_sum_f64(sd);
+  for (int64_t idx = 4 * n4 + t0; idx < total; idx += stride) {
+    const float f = F[idx] * a, p = P[idx] * b;
+    sdf = fmaf(f - p, f - p, sdf);
+    snf = fmaf(f, f, snf);
+  }
+  double sd = block_sum_f64((double)sdf), sn;
   __syncthreads();
-  sn = block_sum_f64(sn);
+  sn = block_sum_f64((double)snf);
   if (threadIdx.x == 0) {
     atomicAdd(d2, sd);
     atomicAdd(n2, sn);
