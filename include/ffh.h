@@ -200,6 +200,40 @@ ffh_status ffh_quad_form(ffh_t h, const void* V, const float* Linv, int64_t N, i
 ffh_status ffh_cholesky(ffh_t h, const float* F, int64_t d, float* L_out, float* Linv_out,
                         double* logdet);
 
+/* ---- WaterKron downstream of the fit (Sections 2-3; device pointers, handle's stream) ---- */
+
+/* Reverse Cholesky (Section 2 notation: RevCholesky(F) is the lower L with L_ii > 0 and
+ * L^T L = F) and the column-normalised inverse used by Algorithms 1-2
+ * (Lt = L^-1 with Lt[:, j] divided by Lt[j][j], so Lt is lower unit-triangular):
+ *   F       d x d fp32 SPD, row-major (read only)
+ *   L_out   d x d fp32 lower (zeros above); nullable
+ *   Lt_out  d x d fp32 lower unit-triangular; nullable
+ *   logdet  host double, log|F|; nullable
+ * Computed as J C^T J from the Cholesky factor C of J F J (J the reversal).
+ * Errors: NOT_SPD, INVALID_ARG, OOM, CUDA. */
+ffh_status ffh_rev_cholesky(ffh_t h, const float* F, int64_t d, float* L_out, float* Lt_out,
+                            double* logdet);
+
+/* Waterfilling scales of Corollary 3.2 (Section 3):
+ *   alpha_j = sqrt(gamma) |A|^(1/2n) / L^A_jj,   beta_i = sqrt(gamma) |B|^(1/2m) / L^B_ii
+ *   LA n x n = RevCholesky(A), LB m x m = RevCholesky(B) (ffh_rev_cholesky); only the
+ *   diagonals are read.  alpha_out n fp32, beta_out m fp32; gamma > 0 sets the rate. */
+ffh_status ffh_waterfilling_scales(ffh_t h, const float* LA, int64_t n, const float* LB, int64_t m,
+                                   float gamma, float* alpha_out, float* beta_out);
+
+/* Two-sided GPTQ quantizer (Algorithm 2): for j = 0..n-1, i = 0..m-1,
+ *   Z_ij = round(W_ij / (alpha_j beta_i)) (nearest, ties to even),
+ *   W <- W + Lt^B[:, i] (alpha_j beta_i Z_ij - W_ij) Lt^A[:, j]^T
+ *   W      m x n fp32, row-major (read only; the feedback goes to a library copy)
+ *   LtA    n x n, LtB m x m: column-normalised inverses from ffh_rev_cholesky
+ *   alpha  n fp32 > 0, beta m fp32 > 0 (e.g. ffh_waterfilling_scales)
+ *   Z_out  m x n int32; V_out m x n fp32 = beta alpha^T (.) Z, nullable
+ * m <= 32768 (one column of feedback per CTA in shared memory).
+ * Errors: INVALID_ARG, OOM, TIMEOUT (a bounded wait between columns expired), CUDA. */
+ffh_status ffh_gptq2(ffh_t h, const float* W, const float* LtA, const float* LtB,
+                     const float* alpha, const float* beta, int64_t m, int64_t n, int32_t* Z_out,
+                     float* V_out);
+
 /* Weighted Gram that allocates no device memory.  The paper has no counterpart: this
  * entry point exists for callers that cannot call cudaMalloc -- code running inside a
  * framework that owns all device memory (a pre-reserved pool, an inference-engine

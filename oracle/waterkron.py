@@ -79,19 +79,36 @@ def gptq2(W: np.ndarray, A: np.ndarray, B: np.ndarray, alpha: np.ndarray,
           beta: np.ndarray) -> np.ndarray:
     """Algorithm 2 (two-sided GPTQ), step by step: for j = 1..n, i = 1..m, round the
     entry and add Lt^B[:, i] Delta Lt^A[:, j]^T to W.  Returns Z (int64)."""
-    W = np.array(W, dtype=np.float64)
-    m, n = W.shape
     LtA = normalized_inverse(rev_cholesky(A))
     LtB = normalized_inverse(rev_cholesky(B))
+    return gptq2_factors(W, LtA, LtB, alpha, beta)
+
+
+def gptq2_factors(W: np.ndarray, LtA: np.ndarray, LtB: np.ndarray, alpha: np.ndarray,
+                  beta: np.ndarray, tie_distance: bool = False):
+    """The loop of Algorithm 2 from its column-normalised inverse factors Lt^A (n x n),
+    Lt^B (m x m).  Returns Z (int64), and with tie_distance also the smallest
+    |frac(W_ij / (alpha_j beta_i)) - 1/2| over the decisions (how far the run stays from
+    a rounding tie, so a comparison in another precision knows whether Z is unique)."""
+    W = np.array(W, dtype=np.float64)
+    LtA = np.asarray(LtA, dtype=np.float64)
+    LtB = np.asarray(LtB, dtype=np.float64)
+    alpha = np.asarray(alpha, dtype=np.float64)
+    beta = np.asarray(beta, dtype=np.float64)
+    m, n = W.shape
     Z = np.zeros((m, n), dtype=np.int64)
+    best = np.inf
     for j in range(n):
         for i in range(m):
-            z = np.rint(W[i, j] / (alpha[j] * beta[i]))
+            t = W[i, j] / (alpha[j] * beta[i])
+            if tie_distance:
+                best = min(best, abs(abs(t - np.floor(t)) - 0.5))
+            z = np.rint(t)
             Z[i, j] = z
             delta = alpha[j] * beta[i] * z - W[i, j]
             # Lt^B[:, i] is zero above row i and Lt^A[:, j] above row j
             W[i:, j:] += delta * np.outer(LtB[i:, i], LtA[j:, j])
-    return Z
+    return (Z, float(best)) if tie_distance else Z
 
 
 def dequantize(Z: np.ndarray, alpha: np.ndarray, beta: np.ndarray) -> np.ndarray:
@@ -104,23 +121,3 @@ def distortion(W: np.ndarray, V: np.ndarray, A: np.ndarray, B: np.ndarray) -> fl
     LA, LB = rev_cholesky(A), rev_cholesky(B)
     E = LB @ (np.asarray(V, np.float64) - np.asarray(W, np.float64)) @ LA.T
     return float(np.sum(E * E) / E.size)
-
-
-def min_tie_distance(W: np.ndarray, A: np.ndarray, B: np.ndarray, alpha: np.ndarray,
-                     beta: np.ndarray) -> float:
-    """Smallest |frac(W_ij / (alpha_j beta_i)) - 1/2| over the decisions of Algorithm 2
-    (same steps as gptq2): how far the run stays from a rounding tie, so a comparison
-    with another precision knows whether its integer result is unique."""
-    W = np.array(W, dtype=np.float64)
-    m, n = W.shape
-    LtA = normalized_inverse(rev_cholesky(A))
-    LtB = normalized_inverse(rev_cholesky(B))
-    best = np.inf
-    for j in range(n):
-        for i in range(m):
-            t = W[i, j] / (alpha[j] * beta[i])
-            best = min(best, abs(abs(t - np.floor(t)) - 0.5))
-            z = np.rint(t)
-            delta = alpha[j] * beta[i] * z - W[i, j]
-            W[i:, j:] += delta * np.outer(LtB[i:, i], LtA[j:, j])
-    return float(best)

@@ -86,6 +86,9 @@ def load_library(path: Optional[str] = None):
         "ffh_weighted_gram_static": ([vp, vp, i64, i64, f32, vp, vp, ctypes.c_char_p, i32],
                                      ctypes.c_int),
         "ffh_phi_tilde": ([vp, vp, vp, i64, i64, i64, vp, vp, pd], ctypes.c_int),
+        "ffh_rev_cholesky": ([vp, vp, i64, vp, vp, pd], ctypes.c_int),
+        "ffh_waterfilling_scales": ([vp, vp, i64, vp, i64, f32, vp, vp], ctypes.c_int),
+        "ffh_gptq2": ([vp, vp, vp, vp, vp, vp, i64, i64, vp, vp], ctypes.c_int),
     }
     for name, (args, res) in sigs.items():
         fn = getattr(lib, name)
@@ -280,6 +283,60 @@ class Handle:
         code = self._lib.ffh_cholesky(self._h, _ptr(F), d, _ptr(L), _ptr(Li), ctypes.byref(ld))
         _check(self._lib, self._h, code, "ffh_cholesky")
         return L, Li, ld.value
+
+    # ---- WaterKron downstream (Sections 2-3) ----
+    def rev_cholesky(self, F: torch.Tensor):
+        """ffh_rev_cholesky: (L with L^T L = F, column-normalised L^-1, log|F|)."""
+        F = F.to(torch.float32).contiguous()
+        d = F.shape[0]
+        L = torch.empty_like(F)
+        Lt = torch.empty_like(F)
+        ld = ctypes.c_double()
+        code = self._lib.ffh_rev_cholesky(self._h, _ptr(F), d, _ptr(L), _ptr(Lt), ctypes.byref(ld))
+        _check(self._lib, self._h, code, "ffh_rev_cholesky")
+        return L, Lt, ld.value
+
+    def waterfilling_scales(self, LA: torch.Tensor, LB: torch.Tensor, gamma: float):
+        """ffh_waterfilling_scales: (alpha, beta) of Corollary 3.2."""
+        LA, LB = LA.to(torch.float32).contiguous(), LB.to(torch.float32).contiguous()
+        n, m = LA.shape[0], LB.shape[0]
+        alpha = torch.empty(n, dtype=torch.float32, device=LA.device)
+        beta = torch.empty(m, dtype=torch.float32, device=LA.device)
+        code = self._lib.ffh_waterfilling_scales(self._h, _ptr(LA), n, _ptr(LB), m, float(gamma),
+                                                 _ptr(alpha), _ptr(beta))
+        _check(self._lib, self._h, code, "ffh_waterfilling_scales")
+        return alpha, beta
+
+    def gptq2(self, W: torch.Tensor, LtA: torch.Tensor, LtB: torch.Tensor, alpha: torch.Tensor,
+              beta: torch.Tensor, want_v: bool = True):
+        """ffh_gptq2 (Algorithm 2): (Z int32, V = beta alpha^T (.) Z or None)."""
+        W = W.to(torch.float32).contiguous()
+        m, n = W.shape
+        Z = torch.empty(m, n, dtype=torch.int32, device=W.device)
+        V = torch.empty(m, n, dtype=torch.float32, device=W.device) if want_v else None
+        args = [t.to(torch.float32).contiguous() for t in (LtA, LtB, alpha, beta)]
+        code = self._lib.ffh_gptq2(self._h, _ptr(W), *[_ptr(t) for t in args], m, n, _ptr(Z),
+                                   _ptr(V))
+        _check(self._lib, self._h, code, "ffh_gptq2")
+        return Z, V
+
+
+def waterkron_quantize(W: torch.Tensor, A: torch.Tensor, B: torch.Tensor, gamma: float,
+                       handle: Optional["Handle"] = None):
+    """Two-sided GPTQ of W (m x n) under A (x) B with the waterfilling scales:
+    RevCholesky(A), RevCholesky(B) -> (alpha, beta) (Corollary 3.2) -> Algorithm 2.
+    Returns (Z, V, alpha, beta)."""
+    own = handle is None
+    h = handle or Handle()
+    try:
+        LA, LtA, _ = h.rev_cholesky(A)
+        LB, LtB, _ = h.rev_cholesky(B)
+        alpha, beta = h.waterfilling_scales(LA, LB, gamma)
+        Z, V = h.gptq2(W, LtA, LtB, alpha, beta)
+        return Z, V, alpha, beta
+    finally:
+        if own:
+            h.close()
 
 
 def weighted_gram_static(V: torch.Tensor, w: Optional[torch.Tensor], scale: float = 1.0,

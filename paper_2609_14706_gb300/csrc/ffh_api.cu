@@ -1002,6 +1002,96 @@ extern "C" ffh_status ffh_cholesky(ffh_t h, const float* F, int64_t d, float* L_
   return es;
 }
 
+extern "C" ffh_status ffh_rev_cholesky(ffh_t h, const float* F, int64_t d, float* L_out,
+                                       float* Lt_out, double* logdet) {
+  if (!h) return FFH_ERR_INVALID_ARG;
+  h->err.clear();
+  if (!F || d < 1) return fail(h, FFH_ERR_INVALID_ARG, "bad arguments");
+  if (!is_device_ptr(F) || (L_out && !is_device_ptr(L_out)) || (Lt_out && !is_device_ptr(Lt_out)))
+    return fail(h, FFH_ERR_INVALID_ARG, "WaterKron calls take device pointers");
+  const int nt = (int)((d + 63) / 64);
+  auto layout = [&](Carve& c, DevStatus** st, float** Fr, float** C, float** Ci, float** work,
+                    float** DI) {
+    *st = c.take<DevStatus>(1);
+    *Fr = c.take<float>((size_t)d * d);
+    *C = c.take<float>((size_t)d * d);
+    *Ci = c.take<float>((size_t)d * d);
+    *work = c.take<float>(std::max(cholesky_work_floats(d), cholesky_tc_work_bytes(d) / 4 + 1));
+    *DI = c.take<float>((size_t)nt * 64 * 64);
+  };
+  DevStatus* st;
+  float *Fr, *C, *Ci, *work, *DI;
+  {
+    Carve c(nullptr);
+    layout(c, &st, &Fr, &C, &Ci, &work, &DI);
+    ffh_status es = ensure_ws(h, c.off + 1024);
+    if (es) return es;
+  }
+  Carve c(h->ws);
+  layout(c, &st, &Fr, &C, &Ci, &work, &DI);
+  cudaStream_t s = h->stream;
+  CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
+  // C C^T = J F J;  L = J C^T J,  L^-1 = J C^-T J (column-normalised for Algorithms 1-2)
+  CK(launch_reverse_sym(F, d, d, Fr, s));
+  ffh_status es = chol(h, Fr, d, C, Ci, work, DI, st,
+                       h->opt.fault == FFH_FAULT_BAD_PIVOT ? FFH_FAULT_BAD_PIVOT : 0);
+  if (es) return es;
+  if (L_out) CK(launch_rev_transpose(C, d, L_out, false, s));
+  if (Lt_out) CK(launch_rev_transpose(Ci, d, Lt_out, true, s));
+  DevStatus hst;
+  CK(cudaMemcpyAsync(&hst, st, sizeof(hst), cudaMemcpyDeviceToHost, s));
+  es = read_status(h, st);
+  if (logdet) *logdet = hst.logdet;
+  return es;
+}
+
+extern "C" ffh_status ffh_waterfilling_scales(ffh_t h, const float* LA, int64_t n, const float* LB,
+                                              int64_t m, float gamma, float* alpha_out,
+                                              float* beta_out) {
+  if (!h) return FFH_ERR_INVALID_ARG;
+  h->err.clear();
+  if (!LA || !LB || !alpha_out || !beta_out || n < 1 || m < 1 || !(gamma > 0.f) ||
+      !std::isfinite(gamma))
+    return fail(h, FFH_ERR_INVALID_ARG, "bad arguments");
+  if (!is_device_ptr(LA) || !is_device_ptr(LB) || !is_device_ptr(alpha_out) ||
+      !is_device_ptr(beta_out))
+    return fail(h, FFH_ERR_INVALID_ARG, "WaterKron calls take device pointers");
+  CK(launch_waterfilling(LA, n, LB, m, gamma, alpha_out, beta_out, h->stream));
+  CK(cudaStreamSynchronize(h->stream));
+  return FFH_OK;
+}
+
+extern "C" ffh_status ffh_gptq2(ffh_t h, const float* W, const float* LtA, const float* LtB,
+                                const float* alpha, const float* beta, int64_t m, int64_t n,
+                                int32_t* Z_out, float* V_out) {
+  if (!h) return FFH_ERR_INVALID_ARG;
+  h->err.clear();
+  if (!W || !LtA || !LtB || !alpha || !beta || !Z_out || m < 1 || n < 1)
+    return fail(h, FFH_ERR_INVALID_ARG, "bad arguments");
+  if (m > 32768) return fail(h, FFH_ERR_INVALID_ARG, "m = %lld > 32768", (long long)m);
+  if (!is_device_ptr(W) || !is_device_ptr(LtA) || !is_device_ptr(LtB) || !is_device_ptr(alpha) ||
+      !is_device_ptr(beta) || !is_device_ptr(Z_out) || (V_out && !is_device_ptr(V_out)))
+    return fail(h, FFH_ERR_INVALID_ARG, "WaterKron calls take device pointers");
+  auto layout = [&](Carve& c, DevStatus** st, void** work) {
+    *st = c.take<DevStatus>(1);
+    *work = c.take<char>(gptq2_work_bytes(m, n));
+  };
+  DevStatus* st;
+  void* work;
+  {
+    Carve c(nullptr);
+    layout(c, &st, &work);
+    ffh_status es = ensure_ws(h, c.off + 1024);
+    if (es) return es;
+  }
+  Carve c(h->ws);
+  layout(c, &st, &work);
+  cudaStream_t s = h->stream;
+  CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
+  CK(launch_gptq2(W, LtA, LtB, alpha, beta, m, n, Z_out, V_out, work, st, s));
+  return read_status(h, st);
+}
+
 extern "C" ffh_status ffh_get_timings(ffh_t h, ffh_timings* out, int32_t reset) {
   if (!h || !out) return FFH_ERR_INVALID_ARG;
   if (!h->pending.empty()) {

@@ -125,6 +125,17 @@ cudaError_t launch_cholesky_tc(const float* F, int64_t d, int64_t ldf, float* L,
                                CholStreams* cs = nullptr);
 size_t cholesky_tc_work_bytes(int64_t d);
 cudaError_t launch_fill_identity(float* F, int64_t d, int64_t ld, cudaStream_t s);
+
+// WaterKron downstream (waterkron.cu)
+cudaError_t launch_reverse_sym(const float* F, int64_t d, int64_t ldf, float* out, cudaStream_t s);
+cudaError_t launch_rev_transpose(const float* C, int64_t d, float* out, bool normalize,
+                                 cudaStream_t s);
+cudaError_t launch_waterfilling(const float* LA, int64_t n, const float* LB, int64_t m,
+                                float gamma, float* alpha, float* beta, cudaStream_t s);
+size_t gptq2_work_bytes(int64_t m, int64_t n);
+cudaError_t launch_gptq2(const float* W, const float* LtA, const float* LtB, const float* alpha,
+                         const float* beta, int64_t m, int64_t n, int32_t* Z, float* V,
+                         void* work, DevStatus* st, cudaStream_t s);
 cudaError_t launch_damp(float* F, int64_t d, int64_t ld, float lambda, DevStatus* st,
                         cudaStream_t s, double* shift_out = nullptr);
 cudaError_t launch_add(float* C, const float* X, int64_t total, cudaStream_t s);

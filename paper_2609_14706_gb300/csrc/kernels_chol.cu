@@ -687,8 +687,9 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
 size_t cholesky_tc_work_bytes(int64_t d) {
   const int64_t kmax = (d + 63) / 64 * 64;
   const int64_t rows = (d + 127) / 128 * 128 + 128;
-  // W copy, T scratch, five split buffers (each <= rows x 2*kmax bf16)
-  return (size_t)d * d * 4 + (size_t)d * d * 4 + 5 * (size_t)rows * 2 * kmax * 2 + 4096;
+  // W copy, T scratch, five split buffers (each <= rows x 2*kmax bf16), each region and the
+  // base rounded up to 256 bytes
+  return (size_t)d * d * 4 + (size_t)d * d * 4 + 5 * (size_t)rows * 2 * kmax * 2 + 8 * 256 + 4096;
 }
 
 cudaError_t chol_streams_init(CholStreams* cs) {
@@ -753,15 +754,19 @@ static cudaError_t cholesky_tc_body(const float* F, int64_t d, int64_t ldf, floa
   cudaError_t e;
   const int64_t kmax = (d + 63) / 64 * 64;
   const int64_t rows_cap = (d + 127) / 128 * 128 + 128;
+  // every region starts on a 256-byte boundary (the split buffers are TMA sources, which
+  // need 16-byte aligned bases; d x d fp32 regions are not multiples of 16 bytes for odd d)
+  auto up = [](size_t b) { return (b + 255) / 256 * 256; };
   char* wp = static_cast<char*>(work);
+  wp = reinterpret_cast<char*>(up(reinterpret_cast<uintptr_t>(wp)));
   float* W = reinterpret_cast<float*>(wp);
-  wp += (size_t)d * d * 4;
+  wp += up((size_t)d * d * 4);
   float* T = reinterpret_cast<float*>(wp);
-  wp += (size_t)d * d * 4;
+  wp += up((size_t)d * d * 4);
   __nv_bfloat16* sb[5];
   for (int i = 0; i < 5; ++i) {
     sb[i] = reinterpret_cast<__nv_bfloat16*>(wp);
-    wp += (size_t)rows_cap * 2 * kmax * 2;
+    wp += up((size_t)rows_cap * 2 * kmax * 2);
   }
   static bool attr = false;
   if (!attr) {

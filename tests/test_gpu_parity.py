@@ -102,8 +102,9 @@ def test_quad_form_matches_oracle(kernel, N, d):
 # Cholesky and inverse
 # ---------------------------------------------------------------------------
 @pytest.mark.parametrize("kernel", KERNELS)
-@pytest.mark.parametrize("d,cond", [(64, 1e2), (200, 1e3), (512, 1e3), (1000, 1e4), (1536, 1e3),
-                                    (2304, 1e3), (4096, 1e4)])
+@pytest.mark.parametrize("d,cond", [(64, 1e2), (129, 1e2), (200, 1e3), (257, 1e3), (512, 1e3),
+                                    (1000, 1e4), (1001, 1e3), (1536, 1e3), (2304, 1e3),
+                                    (4096, 1e4)])
 def test_cholesky_matches_oracle(kernel, d, cond):
     """Cholesky factor L and inverse M = L^-1.  Unit roundoff of the arithmetic:
     CUDA-core path fp32 (u = 2^-24, accumulated over d terms); tensor-core path bf16
