@@ -52,6 +52,8 @@ def parse_args():
     p.add_argument("--seed", type=int, default=0)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-waterkron", action="store_true",
+                   help="skip the WaterKron quantizer timing on the fitted factors")
     p.add_argument("--samples", type=int, default=None,
                    help="override the workload's sample count N (short profiling runs; "
                         "the headline uses the workload's own N)")
@@ -335,6 +337,39 @@ def run_ours(args):
         "gram_frac_of_burst_peak": gram_tflops / float(peaks.get("bf16_tflops")),
     }
 
+    # ---- WaterKron downstream on the fitted factors (Sections 2-3): reverse Cholesky of
+    # A and B, waterfilling scales (Cor. 3.2), two-sided GPTQ (Alg. 2) of a Gaussian
+    # m x n weight matrix
+    waterkron = None
+    if not args.no_waterkron and not matrix:
+        gw = torch.Generator("cuda").manual_seed(args.seed + 99)
+        Wq = torch.randn(m, n, generator=gw, device="cuda")
+        hw = ffh.Handle(stream=stream)
+
+        def factors():
+            LA, LtA, _ = hw.rev_cholesky(A)
+            LB, LtB, _ = hw.rev_cholesky(B)
+            al, be = hw.waterfilling_scales(LA, LB, 0.05)
+            return LtA, LtB, al, be
+
+        LtA, LtB, al, be = factors()
+        hw.gptq2(Wq, LtA, LtB, al, be)  # warm-up
+        w0, w1, w2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+        barrier()
+        w0.record(stream)
+        LtA, LtB, al, be = factors()
+        w1.record(stream)
+        Zq, Vq = hw.gptq2(Wq, LtA, LtB, al, be)
+        w2.record(stream)
+        barrier()
+        waterkron = {"shape_m_n": [m, n], "gamma": 0.05,
+                     "rev_cholesky_and_scales_ms": w0.elapsed_time(w1),
+                     "gptq2_ms": w1.elapsed_time(w2),
+                     "bound": "latency: m n sequential rounding decisions, run as a wavefront "
+                              "of 32-row blocks over 128 columns at a time"}
+        hw.close()
+        del Wq, Zq, Vq
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline and not matrix:
         ns = oracle_sample_size(wl)
@@ -352,7 +387,8 @@ def run_ours(args):
                    "parallelism": f"replicas{world}" if world > 1 else "single",
                    "l2": "inputs (%.1f GB) exceed L2 (129 MB); no flush" %
                          (wl.sample_bytes() / 1e9)},
-        "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e,
+        "roofline": roofline, "kernels": kernels, "waterkron": waterkron, "cpu_baseline": cpu,
+        "e2e": e2e,
         "gpu_launches": int(launches), "clocks": clk,
     }
     if rank == 0:
