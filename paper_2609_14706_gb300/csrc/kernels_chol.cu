@@ -84,12 +84,20 @@ static bool map_bf16_kmajor(CUtensorMap* m, const void* base, uint64_t k_extent,
 //   packed rows z*rows_pad .. of one 2-D buffer.  K' is a list of up to three 64-aligned
 //   segments (x offsets per operand), each kseg wide.
 //   C: fp32 row-major, element (r, c) of batch z at C + z*strideC + r*ldc + c.
+// Epilogue (when C's rows and batches start on 16-byte boundaries): all eight warps take
+// a quarter of the tile's rows (their TMEM lane quarter) and half of its columns; each
+// 32 x 32 block goes TMEM -> registers -> 128-byte-swizzled shared memory -> TMA tensor
+// store, and beta C arrives the same way, loaded by TMA while the MMAs run.  The optional
+// bf16 hi/lo split of the result is staged and stored the same way.  Other C layouts
+// take a per-element epilogue (four warps, rows through a shared transpose).
 // ===========================================================================
 namespace gt {
 constexpr int BM = 128, BN = 128, BK = 64, STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2, B_BYTES = BN * BK * 2;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
+constexpr int BOX_BYTES = 32 * 128;             // one 32-row x 128-byte swizzled box
+constexpr int C_STAGE_BYTES = 16 * BOX_BYTES;   // the fp32 tile as 4 x 4 boxes of 32 x 32
+constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + C_STAGE_BYTES + 256;
 constexpr uint32_t TMEM_COLS = 128;
 }  // namespace gt
 
@@ -105,12 +113,19 @@ struct GemmTcArgs {
   __nv_bfloat16* split_out; // optional: also write the bf16 hi/lo split of the result,
   int split_kpad;           //   row r of batch z at (z*M_pad + r) * 2*split_kpad
   int split_rows_pad;
+  int tma_epi;              // C (and the split) through the tensor maps cmap, hmap, lmap
   DevStatus* st;
 };
 
+// byte offset of 16-byte chunk q of row r in a 128-byte-swizzled box (1024-aligned base)
+__device__ __forceinline__ uint32_t sw128_off(int r, int q) {
+  return (uint32_t)(r * 128 + ((q ^ (r & 7)) << 4));
+}
+
 __global__ void __launch_bounds__(256, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
-              const GemmTcArgs a) {
+              const __grid_constant__ CUtensorMap cmap, const __grid_constant__ CUtensorMap hmap,
+              const __grid_constant__ CUtensorMap lmap, const GemmTcArgs a) {
   using namespace gt;
   pdl_enter();
   const int tn = blockIdx.x, tm = blockIdx.y, z = blockIdx.z;
@@ -119,12 +134,14 @@ __global__ void __launch_bounds__(256, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint8_t* cst = smem + STAGES * STAGE_BYTES;  // C staging (tma_epi)
+  uint64_t* bars = reinterpret_cast<uint64_t*>(cst + C_STAGE_BYTES);
   uint64_t* full = bars;
   uint64_t* empty = bars + STAGES;
   uint64_t* accf = bars + 2 * STAGES;
   uint64_t* drain = accf + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* cbar = drain + 1;  // [8] beta C of each epilogue warp
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(cbar + 8);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   volatile int* skip_flag = abort_flag + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -137,10 +154,23 @@ __global__ void __launch_bounds__(256, 1)
     }
     mbar_init(accf, 1);
     mbar_init(drain, 1);
+    for (int w = 0; w < 8; ++w) mbar_init(&cbar[w], 1);
     fence_mbar_init();
   }
   __syncthreads();
   if (*skip_flag) return;
+  // epilogue geometry (tma_epi): TMEM lane quarter wq, column half ch
+  const int wq = warp & 3, ch = warp >> 2;
+  const bool load_c = a.tma_epi && a.beta != 0.f;
+  if (load_c && lane == 0) {
+    // beta C for this warp's two 32 x 32 blocks, in flight during the MMAs
+    mbar_arrive_expect_tx(&cbar[warp], 2 * BOX_BYTES);
+    for (int h = 0; h < 2; ++h) {
+      const int cb = 2 * ch + h;
+      tma_load_3d(cst + (wq * 4 + cb) * BOX_BYTES, &cmap, &cbar[warp], col0 + 32 * cb,
+                  row0 + 32 * wq, z);
+    }
+  }
   if (warp == 2) {
     tmem_alloc(tmem_slot, TMEM_COLS);
     tmem_relinquish();
@@ -204,8 +234,83 @@ __global__ void __launch_bounds__(256, 1)
     mma_commit(drain);
     volatile int never = 0;
     mbar_wait(drain, 0, &never, kGemmWaitNs);
+  }
+  __syncwarp();
+
+  if (a.tma_epi) {
+    bool ok = mbar_wait(accf, 0, abort_flag, kGemmWaitNs);
+    if (ok && load_c) ok = mbar_wait(&cbar[warp], 0, abort_flag, kGemmWaitNs);
+    if (ok) {
+      tc_fence_after();
+      // every MMA has completed (accf): stages 0-1 hold the split boxes
+      // [hi/lo][column half][lane quarter]
+      uint8_t* hbox = smem + (ch * 4 + wq) * BOX_BYTES;
+      uint8_t* lbox = smem + (8 + ch * 4 + wq) * BOX_BYTES;
+#pragma unroll 1
+      for (int h = 0; h < 2; ++h) {
+        const int cb = 2 * ch + h;
+        uint8_t* cbox = cst + (wq * 4 + cb) * BOX_BYTES;
+        float v[32];
+        tmem_ld32(tmem + ((uint32_t)(wq * 32) << 16) + cb * 32, v);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          float4* cp = reinterpret_cast<float4*>(cbox + sw128_off(lane, q));
+          float4 r;
+          if (load_c) {
+            const float4 pv = *cp;
+            r = make_float4(fmaf(a.beta, pv.x, a.alpha * v[4 * q]),
+                            fmaf(a.beta, pv.y, a.alpha * v[4 * q + 1]),
+                            fmaf(a.beta, pv.z, a.alpha * v[4 * q + 2]),
+                            fmaf(a.beta, pv.w, a.alpha * v[4 * q + 3]));
+          } else {
+            r = make_float4(a.alpha * v[4 * q], a.alpha * v[4 * q + 1], a.alpha * v[4 * q + 2],
+                            a.alpha * v[4 * q + 3]);
+          }
+          *cp = r;
+          v[4 * q] = r.x, v[4 * q + 1] = r.y, v[4 * q + 2] = r.z, v[4 * q + 3] = r.w;
+        }
+        if (a.split_out) {
+          // 32 bf16 = 64 bytes: chunks 4h .. 4h+3 of the row
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            uint32_t hw[4], lw[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float x0 = v[8 * q + 2 * e], x1 = v[8 * q + 2 * e + 1];
+              const __nv_bfloat16 h0 = __float2bfloat16_rn(x0), h1 = __float2bfloat16_rn(x1);
+              const __nv_bfloat16 l0 = __float2bfloat16_rn(x0 - __bfloat162float(h0));
+              const __nv_bfloat16 l1 = __float2bfloat16_rn(x1 - __bfloat162float(h1));
+              hw[e] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+              lw[e] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+            }
+            *reinterpret_cast<uint4*>(hbox + sw128_off(lane, 4 * h + q)) =
+                make_uint4(hw[0], hw[1], hw[2], hw[3]);
+            *reinterpret_cast<uint4*>(lbox + sw128_off(lane, 4 * h + q)) =
+                make_uint4(lw[0], lw[1], lw[2], lw[3]);
+          }
+        }
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        for (int h = 0; h < 2; ++h) {
+          const int cb = 2 * ch + h;
+          tma_store_3d(&cmap, cst + (wq * 4 + cb) * BOX_BYTES, col0 + 32 * cb, row0 + 32 * wq, z);
+        }
+        if (a.split_out) {
+          tma_store_3d(&hmap, hbox, col0 + 64 * ch, row0 + 32 * wq, z);
+          tma_store_3d(&lmap, lbox, col0 + 64 * ch, row0 + 32 * wq, z);
+        }
+        bulk_commit_group();
+        bulk_wait_all();
+      }
+      __syncwarp();
+      tc_fence_before();
+    } else if (lane == 0) {
+      *abort_flag = 1;
+      raise_error(a.st, FFH_ERR_TIMEOUT, 23);
+    }
   } else if (warp >= 4) {
-    const int wq = warp - 4;
     if (mbar_wait(accf, 0, abort_flag, kGemmWaitNs)) {
       tc_fence_after();
       // every MMA has completed (accf), so the stage buffers are free: each warp
@@ -269,18 +374,49 @@ struct Split {
   int batch;
 };
 
+// 3-D tensor map {cols, rows, batch} with 128-byte swizzled boxes of 32 rows x 128 bytes
+// (32 fp32 or 64 bf16 columns); strides in elements.  False where TMA cannot address the
+// layout (bases and strides must be 16-byte multiples).
+static bool map_epi_3d(CUtensorMap* m, const void* base, bool bf16, uint64_t cols,
+                       uint64_t rows, uint64_t batch, uint64_t ld, uint64_t zstride) {
+  const uint64_t es = bf16 ? 2 : 4;
+  if ((reinterpret_cast<uintptr_t>(base) & 15) || (ld * es) % 16) return false;
+  if (batch > 1 && (zstride * es) % 16) return false;
+  auto fn = encode_fn_chol();
+  if (!fn) return false;
+  if (batch == 1) zstride = (rows * ld + 7) / 8 * 8;  // unused; any valid stride
+  cuuint64_t dims[3] = {cols, rows, batch};
+  cuuint64_t strides[2] = {ld * es, zstride * es};
+  cuuint32_t box[3] = {(cuuint32_t)(128 / es), 32, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(m, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3,
+            const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 static cudaError_t gemm_tc(const Split& A, const Split& B, int nseg, const int a_seg[3],
                            const int b_seg[3], int kseg, float* C, int64_t ldc, int64_t strideC,
                            int M, int N, float alpha, float beta, bool lower_only, int batch,
                            DevStatus* st, cudaStream_t s, const Split* out_split = nullptr) {
   if (M <= 0 || N <= 0 || batch <= 0) return cudaSuccess;
-  CUtensorMap am, bm;
+  CUtensorMap am, bm, cm{}, hm{}, lm{};
   if (!map_bf16_kmajor(&am, A.p, (uint64_t)2 * A.kpad, (uint64_t)A.rows_pad * A.batch,
                        (uint64_t)2 * A.kpad, gt::BM))
     return cudaErrorInvalidValue;
   if (!map_bf16_kmajor(&bm, B.p, (uint64_t)2 * B.kpad, (uint64_t)B.rows_pad * B.batch,
                        (uint64_t)2 * B.kpad, gt::BN))
     return cudaErrorInvalidValue;
+  bool tma_epi = map_epi_3d(&cm, C, false, (uint64_t)N, (uint64_t)M, (uint64_t)batch,
+                            (uint64_t)ldc, (uint64_t)strideC);
+  if (tma_epi && out_split) {
+    const uint64_t pitch = (uint64_t)2 * out_split->kpad;
+    const uint64_t zs = (uint64_t)out_split->rows_pad * pitch;
+    tma_epi = map_epi_3d(&hm, out_split->p, true, (uint64_t)N, (uint64_t)M, (uint64_t)batch,
+                         pitch, zs) &&
+              map_epi_3d(&lm, out_split->p + out_split->kpad, true, (uint64_t)N, (uint64_t)M,
+                         (uint64_t)batch, pitch, zs);
+  }
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -308,9 +444,10 @@ static cudaError_t gemm_tc(const Split& A, const Split& B, int nseg, const int a
   g.split_out = out_split ? out_split->p : nullptr;
   g.split_kpad = out_split ? out_split->kpad : 0;
   g.split_rows_pad = out_split ? out_split->rows_pad : 0;
+  g.tma_epi = tma_epi ? 1 : 0;
   g.st = st;
   dim3 grid((N + gt::BN - 1) / gt::BN, (M + gt::BM - 1) / gt::BM, batch);
-  cudaError_t e = launch_pdl(k_gemm_tc, grid, dim3(256), gt::SMEM_BYTES, s, am, bm, g);
+  cudaError_t e = launch_pdl(k_gemm_tc, grid, dim3(256), gt::SMEM_BYTES, s, am, bm, cm, hm, lm, g);
   note_launches(1);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
@@ -363,9 +500,9 @@ static cudaError_t split(const float* src, int64_t lds, int64_t src_stride, int 
 // 128 x 128 diagonal block: Cholesky factor L11 and inverse M11 = L11^-1, one CTA of
 // 512 threads (16 warps), blocked by 32 (sub-panels q = 0..3, rows/cols Q = [32q, 32q+32)).
 //   A(q)  warp 0 factors the 32 x 32 diagonal block D_q and inverts it in registers:
-//         lane i holds row i of D_q and column i of its inverse; pivot j is broadcast
-//         by shuffle, and the remaining columns shift down one register per pivot so
-//         every register index is static.  Writes L_qq, Mi_q = L_qq^-1 and
+//         lane i holds row i of D_q and column i of its inverse; the 2 x 2 pivot block
+//         of columns j, j+1 is broadcast by shuffle, and the remaining columns shift
+//         down two registers per step so every register index is static.  Writes L_qq, Mi_q = L_qq^-1 and
 //         Mt[x][k] = Mi_q[k][x].
 //   B(q)  all warps: the rows below, L[r][Q] = A[r][Q] Mi_q^T (4 x 4 register blocks),
 //         also stored transposed, Pt[k][r] = L[r][32q+k].
@@ -377,8 +514,9 @@ static cudaError_t split(const float* src, int64_t lds, int64_t src_stride, int 
 //         of the next row block (only -Mi_3 T_3 is left after the last sub-panel).
 // Pt and Mt are double-buffered by the parity of q, so A(q+1) never writes what C(q)
 // reads.  The pivot product gives log|F11| = sum_j log(pivot_j).
-// Outputs: L11 and M11 (fp32) and the bf16 hi/lo split of M11 ([hi | lo] rows, pitch
-// 256), the B operand of the panel GEMM.
+// Outputs: L11 and M11 (fp32; their destinations arrive zeroed, so only the lower
+// triangle is stored) and the bf16 hi/lo split of M11 ([hi | lo] rows, pitch 256, dense),
+// the B operand of the panel GEMM.
 // ---------------------------------------------------------------------------
 constexpr int LB = 128;
 constexpr int LP = LB + 1;   // pitch of the row-major 128 x 128 blocks (conflict-free columns)
@@ -387,86 +525,147 @@ constexpr int MP = LB + 4;   // pitch of M11 (float4 rows)
 constexpr int MTP = 36;      // pitch of Mt
 constexpr int TP = 100;      // pitch of the 32 x 96 scratch T
 constexpr int LB_SMEM =
-    (LB * LP + LB * MP + 2 * 32 * PTP + 2 * 32 * MTP + 32 * TP + LB + 64) * 4 + 64;
+    (LB * LP + LB * MP + 2 * 32 * PTP + 2 * 32 * MTP + 32 * TP + LB + 128) * 4 + 64;
 constexpr int LEAF_THREADS = 512;
 
 // A(q): factor and invert the diagonal block (warp 0 only); the pivots go to pivs[c0..].
-// The column of l values of pivot j reaches the other lanes through a shared buffer
-// written rotated (slot (lane - j - 1) mod 32 holds lane lane's value), so the 31 values
-// l_{j+1..j+31, j} are eight broadcast float4 loads; the buffer alternates by the parity of
-// j, so one warp barrier per pivot suffices.  Not inlined: one copy serves the four
-// sub-panels (measured faster than the inlined copies).
+// Two columns per step: every lane forms the 2 x 2 pivot block of columns j, j+1
+// (three shuffles from lanes j, j+1), its own entries l_{lane,j}, l_{lane,j+1} and the
+// matching rows j, j+1 of the inverse, then applies the rank-2 update to its row (and to
+// its column of the inverse) with packed two-wide fp32 FMAs (per component the same
+// rounding as fmaf).  The two updates of an entry are applied one after the other, in
+// the same order and rounding as two one-column steps.  The pairs (l_j, l_{j+1}) reach
+// the other lanes through a shared buffer written rotated (slot s = (lane - j - 2) mod 32
+// holds lane lane's pair), laid out so that one broadcast float4 gives the l_j of slots
+// 2g, 2g+1 followed by their l_{j+1}; the buffer alternates by the parity of j / 2, so one
+// warp barrier per step suffices.  Look-ahead by one step: as soon as step j has updated
+// columns j+2, j+3, the pivot block of step j+2 is factored and its pairs published, and
+// only then does the rest of step j's update run.  Pivot tests are branch-free selects (a
+// failed pivot is replaced by 1 and reported once after the sweep).  Not inlined: one copy
+// serves the four sub-panels.
+struct PivotPair {
+  float l0, l1, m0, m1;
+};
+
+__device__ __forceinline__ PivotPair leaf_pivot_pair(float p00, float p10, float p11, float2 a0,
+                                                     float2 mc0, int j, int c0, float* Ls,
+                                                     float* Ms, float* Mt, float* lbuf,
+                                                     float* pivs, int& first_bad) {
+  const int lane = threadIdx.x & 31;
+  // the tests are warp-uniform (broadcast values)
+  const bool bad0 = !(p00 > 0.f) | !isfinite(p00);
+  p00 = bad0 ? 1.f : p00;
+  // 1/sqrt to within 2 ulp; far below the fp32 accumulation error of the updates
+  const float r0 = rsqrtf(p00);
+  const float l10 = p10 * r0;  // l_{j+1,j}
+  float q11 = fmaf(-l10, l10, p11);
+  const bool bad1 = !(q11 > 0.f) | !isfinite(q11);
+  q11 = bad1 ? 1.f : q11;
+  first_bad = (first_bad < 0 && bad0) ? j : first_bad;
+  first_bad = (first_bad < 0 && bad1) ? j + 1 : first_bad;
+  const float r1 = rsqrtf(q11);
+  PivotPair p;
+  p.l0 = a0.x * r0;                     // lane > j: l_{lane,j}; lane j: sqrt(p00)
+  p.l1 = fmaf(-p.l0, l10, a0.y) * r1;   // lane > j+1: l_{lane,j+1}; lane j+1: diagonal
+  p.m0 = mc0.x * r0;                    // Mi[j][lane]
+  p.m1 = fmaf(-l10, p.m0, mc0.y) * r1;  // Mi[j+1][lane]
+  float* lb = lbuf + ((j >> 1) & 1) * 64;
+  const int slot = (lane - j - 2) & 31;
+  lb[4 * (slot >> 1) + (slot & 1)] = p.l0;
+  lb[4 * (slot >> 1) + 2 + (slot & 1)] = p.l1;
+  if (lane == 0) {
+    pivs[c0 + j] = p00;
+    pivs[c0 + j + 1] = q11;
+  }
+  Ls[(c0 + lane) * LP + c0 + j] = lane >= j ? p.l0 : 0.f;
+  Ls[(c0 + lane) * LP + c0 + j + 1] = lane >= j + 1 ? p.l1 : 0.f;
+  Ms[(c0 + j) * MP + c0 + lane] = p.m0;
+  Ms[(c0 + j + 1) * MP + c0 + lane] = p.m1;
+  *reinterpret_cast<float2*>(Mt + lane * MTP + j) = make_float2(p.m0, p.m1);
+  return p;
+}
+
+// Register pair k of a lane: columns j+2k, j+2k+1 (of its row of D) and rows j+2k, j+2k+1
+// (of its column of the inverse).  Step j's update of pair k (k = 1..15) lands in pair
+// k - 1; v holds (l_j, l_j, l_{j+1}, l_{j+1}) of the two rows j+2k, j+2k+1.
+__device__ __forceinline__ void leaf_pair_update(float2* a2, float2* mc2, int k, float4 v,
+                                                 float2 nl0, float2 nl1, float2 nm0,
+                                                 float2 nm1) {
+  const float2 v0 = make_float2(v.x, v.y), v1 = make_float2(v.z, v.w);
+  a2[k - 1] = __ffma2_rn(nl1, v1, __ffma2_rn(nl0, v0, a2[k]));
+  mc2[k - 1] = __ffma2_rn(v1, nm1, __ffma2_rn(v0, nm0, mc2[k]));
+}
+
 __device__ __noinline__ void leaf_diag(float* Ls, float* Ms, float* Mt, float* lbuf,
                                           float* pivs, int c0, int64_t o, DevStatus* st,
                                           bool& bad) {
   const int lane = threadIdx.x & 31;
   constexpr unsigned FULL = 0xffffffffu;
-  float a[32], mc[32];
+  float2 a2[16], mc2[16];
 #pragma unroll
-  for (int k = 0; k < 32; ++k) {
-    a[k] = (k <= lane) ? Ls[(c0 + lane) * LP + c0 + k] : 0.f;
-    mc[k] = (k == lane) ? 1.f : 0.f;
+  for (int k = 0; k < 16; ++k) {
+    a2[k].x = (2 * k <= lane) ? Ls[(c0 + lane) * LP + c0 + 2 * k] : 0.f;
+    a2[k].y = (2 * k + 1 <= lane) ? Ls[(c0 + lane) * LP + c0 + 2 * k + 1] : 0.f;
+    mc2[k].x = (2 * k == lane) ? 1.f : 0.f;
+    mc2[k].y = (2 * k + 1 == lane) ? 1.f : 0.f;
   }
+  int first_bad = -1;
+  PivotPair p = leaf_pivot_pair(__shfl_sync(FULL, a2[0].x, 0), __shfl_sync(FULL, a2[0].x, 1),
+                                __shfl_sync(FULL, a2[0].y, 1), a2[0], mc2[0], 0, c0, Ls, Ms,
+                                Mt, lbuf, pivs, first_bad);
+  __syncwarp();
 #pragma unroll 1
-  for (int j = 0; j < 32; ++j) {
-    // registers k = 0..31 hold columns j+k of row `lane` (of D) and rows j+k of column
-    // `lane` (of the inverse)
-    float piv = __shfl_sync(FULL, a[0], j);
-    if (!(piv > 0.f) || !isfinite(piv)) {  // warp-uniform (broadcast value)
-      if (lane == 0 && !bad) raise_error(st, FFH_ERR_NOT_SPD, (int)(o + c0 + j));
-      bad = true;
-      piv = 1.f;
-    }
-    // 1/sqrt to within 2 ulp; far below the fp32 accumulation error of the updates
-    const float r = rsqrtf(piv);
-    const float l = a[0] * r;   // lane > j: l_{lane,j}; lane j: sqrt(pivot)
-    const float m = mc[0] * r;  // Mi[j][lane] (exactly 0 for lane > j)
-    float* lb = lbuf + (j & 1) * 32;
-    lb[(lane - j - 1) & 31] = l;
-    if (lane == 0) pivs[c0 + j] = piv;
-    Ls[(c0 + lane) * LP + c0 + j] = lane >= j ? l : 0.f;
-    Ms[(c0 + j) * MP + c0 + lane] = m;
-    Mt[lane * MTP + j] = m;
+  for (int j = 0; j < 30; j += 2) {
+    const float4* lb4 = reinterpret_cast<const float4*>(lbuf + ((j >> 1) & 1) * 64);
+    const float2 nl0 = make_float2(-p.l0, -p.l0), nl1 = make_float2(-p.l1, -p.l1);
+    const float2 nm0 = make_float2(-p.m0, -p.m0), nm1 = make_float2(-p.m1, -p.m1);
+    // pairs past the block (rows j + 2k > 31) only reach registers shifted past the block
+    leaf_pair_update(a2, mc2, 1, lb4[0], nl0, nl1, nm0, nm1);
+    const PivotPair pn = leaf_pivot_pair(
+        __shfl_sync(FULL, a2[0].x, j + 2), __shfl_sync(FULL, a2[0].x, j + 3),
+        __shfl_sync(FULL, a2[0].y, j + 3), a2[0], mc2[0], j + 2, c0, Ls, Ms, Mt, lbuf, pivs,
+        first_bad);
+#pragma unroll
+    for (int k = 2; k < 16; ++k) leaf_pair_update(a2, mc2, k, lb4[k - 1], nl0, nl1, nm0, nm1);
+    a2[15] = make_float2(0.f, 0.f);
+    mc2[15] = make_float2(0.f, 0.f);
+    p = pn;
     __syncwarp();
-    float lk[32];
-#pragma unroll
-    for (int k4 = 0; k4 < 8; ++k4) {
-      const float4 v = *reinterpret_cast<const float4*>(lb + 4 * k4);
-      lk[4 * k4] = v.x;
-      lk[4 * k4 + 1] = v.y;
-      lk[4 * k4 + 2] = v.z;
-      lk[4 * k4 + 3] = v.w;
-    }
-#pragma unroll
-    for (int k = 1; k < 32; ++k) {
-      // lk[k-1] = l_{j+k, j}; for j + k > 31 the value is unused (shifted past the block)
-      a[k - 1] = fmaf(-l, lk[k - 1], a[k]);
-      mc[k - 1] = fmaf(-lk[k - 1], m, mc[k]);
-    }
-    a[31] = 0.f;
-    mc[31] = 0.f;
   }
+  if (first_bad >= 0) {
+    if (lane == 0 && !bad) raise_error(st, FFH_ERR_NOT_SPD, (int)(o + c0 + first_bad));
+    bad = true;
+  }
+}
+
+// acc[0..1] += a * (b.x, b.y), (b.z, b.w): one row of a 4-wide register block in two
+// packed fp32 FMAs (per component the same rounding as fmaf)
+__device__ __forceinline__ void fma_row4(float2* acc, float a, float4 b) {
+  const float2 aa = make_float2(a, a);
+  acc[0] = __ffma2_rn(aa, make_float2(b.x, b.y), acc[0]);
+  acc[1] = __ffma2_rn(aa, make_float2(b.z, b.w), acc[1]);
 }
 
 // Rank-32 update of one 4 x 4 block of the trailing lower triangle from the transposed
 // sub-panel: A[r][c] -= sum_k Pt[k][r] Pt[k][c].
 __device__ __forceinline__ void leaf_trail_block(float* Ls, const float* Pt, int r0, int cc0) {
-  float acc[4][4] = {};
+  float2 acc[4][2] = {};
 #pragma unroll 8
   for (int k = 0; k < 32; ++k) {
     const float4 av = *reinterpret_cast<const float4*>(Pt + k * PTP + r0);
     const float4 bv = *reinterpret_cast<const float4*>(Pt + k * PTP + cc0);
-    const float ar[4] = {av.x, av.y, av.z, av.w}, br[4] = {bv.x, bv.y, bv.z, bv.w};
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-#pragma unroll
-      for (int jx = 0; jx < 4; ++jx) acc[i][jx] = fmaf(ar[i], br[jx], acc[i][jx]);
+    fma_row4(acc[0], av.x, bv);
+    fma_row4(acc[1], av.y, bv);
+    fma_row4(acc[2], av.z, bv);
+    fma_row4(acc[3], av.w, bv);
   }
 #pragma unroll
-  for (int i = 0; i < 4; ++i)
+  for (int i = 0; i < 4; ++i) {
+    const float ac[4] = {acc[i][0].x, acc[i][0].y, acc[i][1].x, acc[i][1].y};
 #pragma unroll
     for (int jx = 0; jx < 4; ++jx)
-      if (cc0 + jx <= r0 + i) Ls[(r0 + i) * LP + cc0 + jx] -= acc[i][jx];
+      if (cc0 + jx <= r0 + i) Ls[(r0 + i) * LP + cc0 + jx] -= ac[jx];
+  }
 }
 
 // Row block Q = [c0, c0 + 32) (c0 >= 32) of the inverse, left of the diagonal block, in
@@ -478,23 +677,17 @@ __device__ __forceinline__ void leaf_inverse_T(const float* Ls, const float* Ms,
   // 2 rows x 4 columns per thread
   for (int blk = t; blk < 16 * nbx; blk += nt) {
     const int i0 = (blk / nbx) * 2, x0 = (blk % nbx) * 4;
-    float acc[2][4] = {};
+    float2 acc[2][2] = {};
     // M lower triangular: M[k][x] = 0 for k < x, so k starts at x0
     for (int k = x0; k < c0; ++k) {
-      float av[2];
-#pragma unroll
-      for (int i = 0; i < 2; ++i) av[i] = Ls[(c0 + i0 + i) * LP + k];
       const float4 bv = *reinterpret_cast<const float4*>(Ms + k * MP + x0);
-      const float br[4] = {bv.x, bv.y, bv.z, bv.w};
 #pragma unroll
-      for (int i = 0; i < 2; ++i)
-#pragma unroll
-        for (int jx = 0; jx < 4; ++jx) acc[i][jx] = fmaf(av[i], br[jx], acc[i][jx]);
+      for (int i = 0; i < 2; ++i) fma_row4(acc[i], Ls[(c0 + i0 + i) * LP + k], bv);
     }
 #pragma unroll
     for (int i = 0; i < 2; ++i)
       *reinterpret_cast<float4*>(T + (i0 + i) * TP + x0) =
-          make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+          make_float4(acc[i][0].x, acc[i][0].y, acc[i][1].x, acc[i][1].y);
   }
 }
 
@@ -504,23 +697,17 @@ __device__ __forceinline__ void leaf_inverse_apply(float* Ms, const float* T, in
   // 2 rows x 4 columns per thread
   for (int blk = t; blk < 16 * nbx; blk += nt) {
     const int i0 = (blk / nbx) * 2, x0 = (blk % nbx) * 4;
-    float acc[2][4] = {};
+    float2 acc[2][2] = {};
     // Mi lower triangular: row i needs j <= i < i0 + 2
     for (int j = 0; j < i0 + 2; ++j) {
-      float av[2];
-#pragma unroll
-      for (int i = 0; i < 2; ++i) av[i] = Ms[(c0 + i0 + i) * MP + c0 + j];
       const float4 bv = *reinterpret_cast<const float4*>(T + j * TP + x0);
-      const float br[4] = {bv.x, bv.y, bv.z, bv.w};
 #pragma unroll
-      for (int i = 0; i < 2; ++i)
-#pragma unroll
-        for (int jx = 0; jx < 4; ++jx) acc[i][jx] = fmaf(av[i], br[jx], acc[i][jx]);
+      for (int i = 0; i < 2; ++i) fma_row4(acc[i], Ms[(c0 + i0 + i) * MP + c0 + j], bv);
     }
 #pragma unroll
     for (int i = 0; i < 2; ++i)
-#pragma unroll
-      for (int jx = 0; jx < 4; ++jx) Ms[(c0 + i0 + i) * MP + x0 + jx] = -acc[i][jx];
+      *reinterpret_cast<float4*>(Ms + (c0 + i0 + i) * MP + x0) =
+          make_float4(-acc[i][0].x, -acc[i][0].y, -acc[i][1].x, -acc[i][1].y);
   }
 }
 
@@ -536,25 +723,35 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
   float* Mtb = Ptb + 2 * 32 * PTP;     // [2][32][MTP] transposed diagonal-block inverses
   float* T = Mtb + 2 * 32 * MTP;       // [32][TP]
   float* pivs = T + 32 * TP;           // [LB] pivots
-  float* lbuf = pivs + LB;             // [2][32] pivot-column broadcast (warp 0)
+  float* lbuf = pivs + LB;             // [2][32][2] pivot-column pair broadcast (warp 0)
   pdl_enter();
   const int b = (int)((d - o) < LB ? (d - o) : LB);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  for (int idx = tid; idx < LB * LB / 4; idx += LEAF_THREADS) {
+  // the lower triangle of the block, all loads of a thread in flight together
+  constexpr int NLD = LB * LB / 4 / LEAF_THREADS;
+  float4 v[NLD];
+#pragma unroll
+  for (int u = 0; u < NLD; ++u) {
+    const int idx = tid + u * LEAF_THREADS;
     const int i = idx >> 5, j4 = (idx & 31) * 4;
-    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (i < b) {
+    v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (i < b && j4 <= i) {
       const float* src = W + (o + i) * ldw + o + j4;
       if (j4 + 3 < b && (((uintptr_t)src) & 15) == 0) {
-        v = *reinterpret_cast<const float4*>(src);
+        v[u] = *reinterpret_cast<const float4*>(src);
       } else {
-        if (j4 + 0 < b) v.x = src[0];
-        if (j4 + 1 < b) v.y = src[1];
-        if (j4 + 2 < b) v.z = src[2];
-        if (j4 + 3 < b) v.w = src[3];
+        if (j4 + 0 < b) v[u].x = src[0];
+        if (j4 + 1 < b) v[u].y = src[1];
+        if (j4 + 2 < b) v[u].z = src[2];
+        if (j4 + 3 < b) v[u].w = src[3];
       }
     }
-    const float vv[4] = {v.x, v.y, v.z, v.w};
+  }
+#pragma unroll
+  for (int u = 0; u < NLD; ++u) {
+    const int idx = tid + u * LEAF_THREADS;
+    const int i = idx >> 5, j4 = (idx & 31) * 4;
+    const float vv[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
       const int j = j4 + e;
@@ -581,22 +778,22 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
     const int R = LB - c0 - 32;
     const bool has = tid < (R / 4) * 8;
     const int r0 = c0 + 32 + (tid >> 3) * 4, k0 = (tid & 7) * 4;
-    float acc[4][4] = {};
+    float2 acc2[4][2] = {};
     if (has) {
       for (int x = 0; x < k0 + 4; ++x) {  // Mi[k][x] = 0 for x > k
-        float av[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) av[i] = Ls[(r0 + i) * LP + c0 + x];
         const float4 bv = *reinterpret_cast<const float4*>(Mt + x * MTP + k0);
-        const float br[4] = {bv.x, bv.y, bv.z, bv.w};
 #pragma unroll
-        for (int i = 0; i < 4; ++i)
-#pragma unroll
-          for (int jx = 0; jx < 4; ++jx) acc[i][jx] = fmaf(av[i], br[jx], acc[i][jx]);
+        for (int i = 0; i < 4; ++i) fma_row4(acc2[i], Ls[(r0 + i) * LP + c0 + x], bv);
       }
     }
     __syncthreads();
     if (has) {
+      float acc[4][4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        acc[i][0] = acc2[i][0].x, acc[i][1] = acc2[i][0].y;
+        acc[i][2] = acc2[i][1].x, acc[i][3] = acc2[i][1].y;
+      }
 #pragma unroll
       for (int i = 0; i < 4; ++i)
 #pragma unroll
@@ -650,7 +847,8 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
       lv[e] = (j <= i) ? Ls[i * LP + j] : 0.f;
       mv[e] = (j <= i && i < b && j < b) ? Ms[i * MP + j] : 0.f;
     }
-    if (i < b) {
+    // L and Minv arrive zeroed: groups entirely above the diagonal are not stored
+    if (i < b && j0 <= i) {
       if (vec_ok && j0 + 3 < b) {
         *reinterpret_cast<float4*>(L + (o + i) * ldl + o + j0) = make_float4(lv[0], lv[1], lv[2], lv[3]);
         *reinterpret_cast<float4*>(Minv + (o + i) * ldm + o + j0) =
