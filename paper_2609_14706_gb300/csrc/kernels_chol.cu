@@ -302,7 +302,7 @@ __global__ void __launch_bounds__(256, 1)
           tma_store_3d(&lmap, lbox, col0 + 64 * ch, row0 + 32 * wq, z);
         }
         bulk_commit_group();
-        bulk_wait_all();
+        bulk_wait_read_all();
       }
       __syncwarp();
       tc_fence_before();
@@ -460,38 +460,58 @@ static cudaError_t gemm_tc(const Split& A, const Split& B, int nseg, const int a
 //   dst[(z*rows_pad + r)*2kpad + c] = hi, [... + kpad + c] = lo; zero elsewhere up to
 //   rows_pad x 2kpad.
 // ---------------------------------------------------------------------------
-__global__ void k_split_hilo(const float* __restrict__ src, int64_t lds, int64_t src_stride,
-                             int rows, int cols, int trans, __nv_bfloat16* __restrict__ dst,
-                             int rows_pad, int kpad, int batch) {
+// One 64 x 64 tile of (r, c) per block, staged through shared memory so that the source
+// is read along its contiguous dimension in both orientations; each thread then writes
+// four consecutive columns of hi and of lo (8 bytes each).
+constexpr int SPLIT_TILE = 64;
+__global__ void __launch_bounds__(256) k_split_hilo(const float* __restrict__ src, int64_t lds,
+                                                    int64_t src_stride, int rows, int cols,
+                                                    int trans, __nv_bfloat16* __restrict__ dst,
+                                                    int rows_pad, int kpad) {
   pdl_enter();
-  const int64_t per = (int64_t)rows_pad * kpad;
-  const int64_t total = per * batch;
-  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
-       idx += (int64_t)gridDim.x * blockDim.x) {
-    const int z = (int)(idx / per);
-    const int64_t rem = idx - (int64_t)z * per;
-    const int r = (int)(rem / kpad), c = (int)(rem - (int64_t)r * kpad);
-    float x = 0.f;
-    if (r < rows && c < cols) {
-      const float* sz = src + (int64_t)z * src_stride;
-      x = trans ? sz[(int64_t)c * lds + r] : sz[(int64_t)r * lds + c];
+  __shared__ float tile[SPLIT_TILE][SPLIT_TILE + 1];
+  const int z = blockIdx.z;
+  const int r0 = blockIdx.y * SPLIT_TILE, c0 = blockIdx.x * SPLIT_TILE;
+  const float* sz = src + (int64_t)z * src_stride;
+  const int t = threadIdx.x;
+  const int f = t & 63, g = t >> 6;  // fast (contiguous) and slow index of the source read
+#pragma unroll 4
+  for (int i = 0; i < SPLIT_TILE / 4; ++i) {
+    const int sl = g + 4 * i;
+    if (!trans) {
+      const int r = r0 + sl, c = c0 + f;
+      tile[sl][f] = (r < rows && c < cols) ? sz[(int64_t)r * lds + c] : 0.f;
+    } else {
+      const int r = r0 + f, c = c0 + sl;  // view (r, c) = source row c, column r
+      tile[f][sl] = (r < rows && c < cols) ? sz[(int64_t)c * lds + r] : 0.f;
     }
-    const __nv_bfloat16 hi = __float2bfloat16_rn(x);
-    const __nv_bfloat16 lo = __float2bfloat16_rn(x - __bfloat162float(hi));
-    __nv_bfloat16* drow = dst + ((int64_t)z * rows_pad + r) * (2 * (int64_t)kpad);
-    drow[c] = hi;
-    drow[kpad + c] = lo;
+  }
+  __syncthreads();
+  const int cq = (t & 15) * 4;
+#pragma unroll 4
+  for (int i = 0; i < SPLIT_TILE / 16; ++i) {
+    const int rr = (t >> 4) + 16 * i;
+    __nv_bfloat16 hi[4], lo[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float x = tile[rr][cq + e];
+      hi[e] = __float2bfloat16_rn(x);
+      lo[e] = __float2bfloat16_rn(x - __bfloat162float(hi[e]));
+    }
+    __nv_bfloat16* drow = dst + ((int64_t)z * rows_pad + r0 + rr) * (2 * (int64_t)kpad);
+    *reinterpret_cast<uint2*>(drow + c0 + cq) = *reinterpret_cast<const uint2*>(hi);
+    *reinterpret_cast<uint2*>(drow + kpad + c0 + cq) = *reinterpret_cast<const uint2*>(lo);
   }
 }
 
 static cudaError_t split(const float* src, int64_t lds, int64_t src_stride, int rows, int cols,
                          bool trans, const Split& d, cudaStream_t s) {
-  const int64_t total = (int64_t)d.rows_pad * d.kpad * d.batch;
-  if (total == 0) return cudaSuccess;
-  const int64_t blocks = std::min<int64_t>((total + 255) / 256, (int64_t)num_sms() * 16);
-  cudaError_t e = launch_pdl(k_split_hilo, dim3((unsigned)blocks), dim3(256), 0, s, src, lds,
-                             src_stride, rows, cols, trans ? 1 : 0, d.p, d.rows_pad, d.kpad,
-                             d.batch);
+  if ((int64_t)d.rows_pad * d.kpad * d.batch == 0) return cudaSuccess;
+  // rows_pad (a multiple of 128) and kpad (a multiple of 64) are whole tiles
+  const dim3 grid((unsigned)(d.kpad / SPLIT_TILE), (unsigned)(d.rows_pad / SPLIT_TILE),
+                  (unsigned)d.batch);
+  cudaError_t e = launch_pdl(k_split_hilo, grid, dim3(256), 0, s, src, lds, src_stride, rows,
+                             cols, trans ? 1 : 0, d.p, d.rows_pad, d.kpad);
   note_launches(1);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
@@ -524,9 +544,16 @@ constexpr int PTP = LB + 4;  // pitch of Pt (float4 rows)
 constexpr int MP = LB + 4;   // pitch of M11 (float4 rows)
 constexpr int MTP = 36;      // pitch of Mt
 constexpr int TP = 100;      // pitch of the 32 x 96 scratch T
-constexpr int LB_SMEM =
-    (LB * LP + LB * MP + 2 * 32 * PTP + 2 * 32 * MTP + 32 * TP + LB + 128) * 4 + 64;
 constexpr int LEAF_THREADS = 512;
+// float offsets of the regions of the kernel's dynamic shared memory
+constexpr int OFF_LS = 0;                          // [LB][LP]  working block -> L11
+constexpr int OFF_MS = OFF_LS + LB * LP;           // [LB][MP]  M11
+constexpr int OFF_PT = OFF_MS + LB * MP;           // [2][32][PTP] transposed sub-panels
+constexpr int OFF_MT = OFF_PT + 2 * 32 * PTP;      // [2][32][MTP] diagonal-block inverses^T
+constexpr int OFF_T = OFF_MT + 2 * 32 * MTP;       // [32][TP]
+constexpr int OFF_PIV = OFF_T + 32 * TP;           // [LB] pivots
+constexpr int OFF_LBUF = OFF_PIV + LB;             // [2][32][2] pair broadcast (warp 0)
+constexpr int LB_SMEM = (OFF_LBUF + 128) * 4 + 64;
 
 // A(q): factor and invert the diagonal block (warp 0 only); the pivots go to pivs[c0..].
 // Two columns per step: every lane forms the 2 x 2 pivot block of columns j, j+1
@@ -539,50 +566,59 @@ constexpr int LEAF_THREADS = 512;
 // holds lane lane's pair), laid out so that one broadcast float4 gives the l_j of slots
 // 2g, 2g+1 followed by their l_{j+1}; the buffer alternates by the parity of j / 2, so one
 // warp barrier per step suffices.  Look-ahead by one step: as soon as step j has updated
-// columns j+2, j+3, the pivot block of step j+2 is factored and its pairs published, and
-// only then does the rest of step j's update run.  Pivot tests are branch-free selects (a
-// failed pivot is replaced by 1 and reported once after the sweep).  Not inlined: one copy
-// serves the four sub-panels.
+// columns j+2, j+3, the pivot block of step j+2 is factored in registers while the rest
+// of step j's update runs, and published (stores) after it, so the pivot chain (shuffles,
+// two reciprocal square roots) overlaps the update.  Pivot tests are branch-free selects
+// (a failed pivot is replaced by 1 and reported once after the sweep).  Not inlined: one
+// copy serves the four sub-panels.
 struct PivotPair {
-  float l0, l1, m0, m1;
+  float l0, l1, m0, m1, p00, q11;
+  bool bad0, bad1;
 };
 
+// The 2 x 2 pivot block of columns j, j+1 and this lane's entries (registers only).
 __device__ __forceinline__ PivotPair leaf_pivot_pair(float p00, float p10, float p11, float2 a0,
-                                                     float2 mc0, int j, int c0, float* Ls,
-                                                     float* Ms, float* Mt, float* lbuf,
-                                                     float* pivs, int& first_bad) {
-  const int lane = threadIdx.x & 31;
+                                                     float2 mc0) {
+  PivotPair p;
   // the tests are warp-uniform (broadcast values)
-  const bool bad0 = !(p00 > 0.f) | !isfinite(p00);
-  p00 = bad0 ? 1.f : p00;
+  p.bad0 = !(p00 > 0.f) | !isfinite(p00);
+  p00 = p.bad0 ? 1.f : p00;
   // 1/sqrt to within 2 ulp; far below the fp32 accumulation error of the updates
   const float r0 = rsqrtf(p00);
   const float l10 = p10 * r0;  // l_{j+1,j}
   float q11 = fmaf(-l10, l10, p11);
-  const bool bad1 = !(q11 > 0.f) | !isfinite(q11);
-  q11 = bad1 ? 1.f : q11;
-  first_bad = (first_bad < 0 && bad0) ? j : first_bad;
-  first_bad = (first_bad < 0 && bad1) ? j + 1 : first_bad;
+  p.bad1 = !(q11 > 0.f) | !isfinite(q11);
+  q11 = p.bad1 ? 1.f : q11;
   const float r1 = rsqrtf(q11);
-  PivotPair p;
+  p.p00 = p00;
+  p.q11 = q11;
   p.l0 = a0.x * r0;                     // lane > j: l_{lane,j}; lane j: sqrt(p00)
   p.l1 = fmaf(-p.l0, l10, a0.y) * r1;   // lane > j+1: l_{lane,j+1}; lane j+1: diagonal
   p.m0 = mc0.x * r0;                    // Mi[j][lane]
   p.m1 = fmaf(-l10, p.m0, mc0.y) * r1;  // Mi[j+1][lane]
+  return p;
+}
+
+// Publish step j's pair: the rotated broadcast buffer, L, M11, Mt and the pivots.
+__device__ __forceinline__ void leaf_pivot_store(const PivotPair& p, int j, int c0, float* Ls,
+                                                 float* Ms, float* Mt, float* lbuf, float* pivs,
+                                                 int& first_bad) {
+  const int lane = threadIdx.x & 31;
+  first_bad = (first_bad < 0 && p.bad0) ? j : first_bad;
+  first_bad = (first_bad < 0 && p.bad1) ? j + 1 : first_bad;
   float* lb = lbuf + ((j >> 1) & 1) * 64;
   const int slot = (lane - j - 2) & 31;
   lb[4 * (slot >> 1) + (slot & 1)] = p.l0;
   lb[4 * (slot >> 1) + 2 + (slot & 1)] = p.l1;
   if (lane == 0) {
-    pivs[c0 + j] = p00;
-    pivs[c0 + j + 1] = q11;
+    pivs[c0 + j] = p.p00;
+    pivs[c0 + j + 1] = p.q11;
   }
   Ls[(c0 + lane) * LP + c0 + j] = lane >= j ? p.l0 : 0.f;
   Ls[(c0 + lane) * LP + c0 + j + 1] = lane >= j + 1 ? p.l1 : 0.f;
   Ms[(c0 + j) * MP + c0 + lane] = p.m0;
   Ms[(c0 + j + 1) * MP + c0 + lane] = p.m1;
   *reinterpret_cast<float2*>(Mt + lane * MTP + j) = make_float2(p.m0, p.m1);
-  return p;
 }
 
 // Register pair k of a lane: columns j+2k, j+2k+1 (of its row of D) and rows j+2k, j+2k+1
@@ -596,9 +632,16 @@ __device__ __forceinline__ void leaf_pair_update(float2* a2, float2* mc2, int k,
   mc2[k - 1] = __ffma2_rn(v1, nm1, __ffma2_rn(v0, nm0, mc2[k]));
 }
 
-__device__ __noinline__ void leaf_diag(float* Ls, float* Ms, float* Mt, float* lbuf,
-                                          float* pivs, int c0, int64_t o, DevStatus* st,
+__device__ __noinline__ void leaf_diag(int mt_off, int c0, int64_t o, DevStatus* st,
                                           bool& bad) {
+  // the regions are addressed from the kernel's shared array (not through pointer
+  // arguments), so every access compiles to a shared-memory instruction
+  extern __shared__ float sh[];
+  float* Ls = sh + OFF_LS;
+  float* Ms = sh + OFF_MS;
+  float* Mt = sh + mt_off;
+  float* lbuf = sh + OFF_LBUF;
+  float* pivs = sh + OFF_PIV;
   const int lane = threadIdx.x & 31;
   constexpr unsigned FULL = 0xffffffffu;
   float2 a2[16], mc2[16];
@@ -611,8 +654,8 @@ __device__ __noinline__ void leaf_diag(float* Ls, float* Ms, float* Mt, float* l
   }
   int first_bad = -1;
   PivotPair p = leaf_pivot_pair(__shfl_sync(FULL, a2[0].x, 0), __shfl_sync(FULL, a2[0].x, 1),
-                                __shfl_sync(FULL, a2[0].y, 1), a2[0], mc2[0], 0, c0, Ls, Ms,
-                                Mt, lbuf, pivs, first_bad);
+                                __shfl_sync(FULL, a2[0].y, 1), a2[0], mc2[0]);
+  leaf_pivot_store(p, 0, c0, Ls, Ms, Mt, lbuf, pivs, first_bad);
   __syncwarp();
 #pragma unroll 1
   for (int j = 0; j < 30; j += 2) {
@@ -621,14 +664,17 @@ __device__ __noinline__ void leaf_diag(float* Ls, float* Ms, float* Mt, float* l
     const float2 nm0 = make_float2(-p.m0, -p.m0), nm1 = make_float2(-p.m1, -p.m1);
     // pairs past the block (rows j + 2k > 31) only reach registers shifted past the block
     leaf_pair_update(a2, mc2, 1, lb4[0], nl0, nl1, nm0, nm1);
-    const PivotPair pn = leaf_pivot_pair(
-        __shfl_sync(FULL, a2[0].x, j + 2), __shfl_sync(FULL, a2[0].x, j + 3),
-        __shfl_sync(FULL, a2[0].y, j + 3), a2[0], mc2[0], j + 2, c0, Ls, Ms, Mt, lbuf, pivs,
-        first_bad);
+    // step j+2's pivot block, in registers only: no shared-memory store comes between the
+    // broadcast loads below and the chain, so the two overlap
+    const PivotPair pn =
+        leaf_pivot_pair(__shfl_sync(FULL, a2[0].x, j + 2), __shfl_sync(FULL, a2[0].x, j + 3),
+                        __shfl_sync(FULL, a2[0].y, j + 3), a2[0], mc2[0]);
 #pragma unroll
     for (int k = 2; k < 16; ++k) leaf_pair_update(a2, mc2, k, lb4[k - 1], nl0, nl1, nm0, nm1);
     a2[15] = make_float2(0.f, 0.f);
     mc2[15] = make_float2(0.f, 0.f);
+    // every lane has read step j's buffer; step j+2 writes the other one
+    leaf_pivot_store(pn, j + 2, c0, Ls, Ms, Mt, lbuf, pivs, first_bad);
     p = pn;
     __syncwarp();
   }
@@ -717,13 +763,12 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
                                                                __nv_bfloat16* m11_split,
                                                                DevStatus* st, int fault) {
   extern __shared__ float sh[];
-  float* Ls = sh;                      // [LB][LP]  working block -> L11
-  float* Ms = Ls + LB * LP;            // [LB][MP]  M11
-  float* Ptb = Ms + LB * MP;           // [2][32][PTP] transposed sub-panels
-  float* Mtb = Ptb + 2 * 32 * PTP;     // [2][32][MTP] transposed diagonal-block inverses
-  float* T = Mtb + 2 * 32 * MTP;       // [32][TP]
-  float* pivs = T + 32 * TP;           // [LB] pivots
-  float* lbuf = pivs + LB;             // [2][32][2] pivot-column pair broadcast (warp 0)
+  float* Ls = sh + OFF_LS;
+  float* Ms = sh + OFF_MS;
+  float* Ptb = sh + OFF_PT;
+  float* Mtb = sh + OFF_MT;
+  float* T = sh + OFF_T;
+  float* pivs = sh + OFF_PIV;
   pdl_enter();
   const int b = (int)((d - o) < LB ? (d - o) : LB);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -765,7 +810,7 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
   if (tid == 0 && fault == FFH_FAULT_BAD_PIVOT && o == 0) Ls[0] = __int_as_float(0x7fc00000);
   __syncthreads();
   bool bad = false;
-  if (warp == 0) leaf_diag(Ls, Ms, Mtb, lbuf, pivs, 0, o, st, bad);
+  if (warp == 0) leaf_diag(OFF_MT, 0, o, st, bad);
   __syncthreads();
 #pragma unroll 1
   for (int q = 0; q < 4; ++q) {
@@ -812,7 +857,7 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
         if (bj <= bi) leaf_trail_block(Ls, Pt, c0 + 32 + 4 * bi, c0 + 32 + 4 * bj);
         asm volatile("bar.sync 1, 64;" ::: "memory");
         if (warp == 0)
-          leaf_diag(Ls, Ms, Mtb + ((q + 1) & 1) * 32 * MTP, lbuf, pivs, c0 + 32, o, st, bad);
+          leaf_diag(OFF_MT + ((q + 1) & 1) * 32 * MTP, c0 + 32, o, st, bad);
       } else if (warp & 3) {
         // warps 2, 3, 5-7, 9-11, 13-15: warps 4, 8 and 12 stay idle so that warp 0's
         // pivot chain has its scheduler partition to itself

@@ -101,9 +101,10 @@ __device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void*
 __device__ __forceinline__ void bulk_commit_group() {
   asm volatile("cp.async.bulk.commit_group;" ::: "memory");
 }
-// all of this thread's committed bulk stores have completed (writes performed)
-__device__ __forceinline__ void bulk_wait_all() {
-  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+// all of this thread's committed bulk stores have finished reading shared memory (the
+// writes to global memory complete before the grid does)
+__device__ __forceinline__ void bulk_wait_read_all() {
+  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
 // generic-proxy shared-memory writes -> visible to the async proxy (tcgen05.mma reads)
 __device__ __forceinline__ void fence_proxy_async_smem() {
