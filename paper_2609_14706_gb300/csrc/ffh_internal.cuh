@@ -80,7 +80,8 @@ cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t
                            const GramPlan& plan, DevStatus* st, int fault, cudaStream_t s,
                            cudaEvent_t after_main = nullptr, const __nv_bfloat16* Va = nullptr,
                            int64_t lda = 0);
-// Vw[k][:] = bf16(w_k V[k][:]), bf16 rows of d (multiple of 8) elements, 16-byte aligned
+// Vw[k][:] = bf16(w_k V[k][:]), bf16 rows of d elements (pitches multiples of 8 elements,
+// 16-byte aligned; the padding up to the next multiple of 8 is written too)
 cudaError_t launch_scale_rows(const __nv_bfloat16* V, int64_t ld, int64_t N, int64_t d,
                               const float* w, __nv_bfloat16* Vw, int64_t ldw, cudaStream_t s);
 // q_k = ||M v_k||^2, V bf16 N x d (pitch ld), M bf16 d x d lower (pitch ldm)

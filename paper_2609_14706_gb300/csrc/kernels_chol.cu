@@ -114,8 +114,14 @@ struct GemmTcArgs {
   int split_kpad;           //   row r of batch z at (z*M_pad + r) * 2*split_kpad
   int split_rows_pad;
   int tma_epi;              // C (and the split) through the tensor maps cmap, hmap, lmap
+  int tri;                  // TRI_* : K blocks a tile can skip (exact zeros of a triangle)
   DevStatus* st;
 };
+// A triangular operand makes part of each tile's K range exact zeros: with
+// TRI_K_FROM_COL, B'[c][k] = 0 for k < c (B' upper), so a tile needs k >= col0; with
+// TRI_K_TO_ROW, A'[r][k] = 0 for k > r (A' lower), so it needs k < row0 + BM.  The skipped
+// 64-blocks contribute nothing, so every tile keeps at least one block.
+constexpr int TRI_K_FROM_COL = 1, TRI_K_TO_ROW = 2;
 
 // byte offset of 16-byte chunk q of row r in a 128-byte-swizzled box (1024-aligned base)
 __device__ __forceinline__ uint32_t sw128_off(int r, int q) {
@@ -179,7 +185,12 @@ __global__ void __launch_bounds__(256, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const int nk = a.nseg * a.kseg_blocks;
+  int kb_lo = (a.tri & TRI_K_FROM_COL) ? col0 / BK : 0;
+  int kb_hi = a.kseg_blocks;
+  if (a.tri & TRI_K_TO_ROW) kb_hi = min(kb_hi, (row0 + BM + BK - 1) / BK);
+  if (kb_lo > kb_hi - 1) kb_lo = kb_hi - 1;
+  const int nkb = kb_hi - kb_lo;  // 64-blocks of each segment
+  const int nk = a.nseg * nkb;
   const int arow = z * a.a_rows_pad + row0, brow = z * a.b_rows_pad + col0;
 
   if (warp == 0 && lane == 0) {
@@ -192,7 +203,7 @@ __global__ void __launch_bounds__(256, 1)
         ok = false;
         break;
       }
-      const int seg = it / a.kseg_blocks, kb = it - seg * a.kseg_blocks;
+      const int seg = it / nkb, kb = kb_lo + it - seg * nkb;
       mbar_arrive_expect_tx(&full[s], STAGE_BYTES);
       uint8_t* sa = smem + s * STAGE_BYTES;
       tma_load_2d(sa, &amap, &full[s], a.a_off[seg] + kb * BK, arow);
@@ -398,7 +409,8 @@ static bool map_epi_3d(CUtensorMap* m, const void* base, bool bf16, uint64_t col
 static cudaError_t gemm_tc(const Split& A, const Split& B, int nseg, const int a_seg[3],
                            const int b_seg[3], int kseg, float* C, int64_t ldc, int64_t strideC,
                            int M, int N, float alpha, float beta, bool lower_only, int batch,
-                           DevStatus* st, cudaStream_t s, const Split* out_split = nullptr) {
+                           DevStatus* st, cudaStream_t s, const Split* out_split = nullptr,
+                           int tri = 0) {
   if (M <= 0 || N <= 0 || batch <= 0) return cudaSuccess;
   CUtensorMap am, bm, cm{}, hm{}, lm{};
   if (!map_bf16_kmajor(&am, A.p, (uint64_t)2 * A.kpad, (uint64_t)A.rows_pad * A.batch,
@@ -445,6 +457,7 @@ static cudaError_t gemm_tc(const Split& A, const Split& B, int nseg, const int a
   g.split_kpad = out_split ? out_split->kpad : 0;
   g.split_rows_pad = out_split ? out_split->rows_pad : 0;
   g.tma_epi = tma_epi ? 1 : 0;
+  g.tri = tri;
   g.st = st;
   dim3 grid((N + gt::BN - 1) / gt::BN, (M + gt::BM - 1) / gt::BM, batch);
   cudaError_t e = launch_pdl(k_gemm_tc, grid, dim3(256), gt::SMEM_BYTES, s, am, bm, cm, hm, lm, g);
@@ -1107,8 +1120,9 @@ static cudaError_t cholesky_tc_body(const float* F, int64_t d, int64_t ldf, floa
       if ((e = split(Linv + o * d + o, d, zs, (int)b, (int)b, true, m11t, s)) != cudaSuccess)
         return e;
       const int as1[3] = {0, 0, kb}, bs1[3] = {0, kb, 0};
+      // B' = M11^T is upper triangular: output column block c needs k >= c
       if ((e = gemm_tc(l21, m11t, 3, as1, bs1, (int)b, T, b, (int64_t)rp * b, rows, (int)b, 1.f,
-                       0.f, false, batch, st, s)) != cudaSuccess)
+                       0.f, false, batch, st, s, nullptr, TRI_K_FROM_COL)) != cudaSuccess)
         return e;
       // M21_z = -M22_z T_z : A' = split(M22) (rows x rows), B' = split(T^T) (b x rows)
       Split m22{sb[2], rp, kr, batch};
@@ -1119,8 +1133,9 @@ static cudaError_t cholesky_tc_body(const float* F, int64_t d, int64_t ldf, floa
       // B'[c][k] = T[k][c]: b output rows, `rows` output columns
       if ((e = split(T, b, (int64_t)rp * b, (int)b, rows, true, tt, s)) != cudaSuccess) return e;
       const int as2[3] = {0, 0, kr}, bs2[3] = {0, kr, 0};
+      // A' = M22 is lower triangular: output row block r needs k < r + 128
       if ((e = gemm_tc(m22, tt, 3, as2, bs2, rows, Linv + (o + b) * d + o, d, zs, rows, (int)b,
-                       -1.f, 0.f, false, batch, st, s)) != cudaSuccess)
+                       -1.f, 0.f, false, batch, st, s, nullptr, TRI_K_TO_ROW)) != cudaSuccess)
         return e;
     }
   }

@@ -473,13 +473,15 @@ __global__ void k_scale_rows(const __nv_bfloat16* __restrict__ V, int64_t ld, in
 
 cudaError_t launch_scale_rows(const __nv_bfloat16* V, int64_t ld, int64_t N, int64_t d,
                               const float* w, __nv_bfloat16* Vw, int64_t ldw, cudaStream_t s) {
-  if (d % 8 || ld % 8 || ldw % 8 ||
-      ((reinterpret_cast<uintptr_t>(V) | reinterpret_cast<uintptr_t>(Vw)) & 15))
+  // rows are processed in 8-element chunks up to the padded width (the pitches are
+  // multiples of 8); the padding columns are never read as operands
+  if (ld % 8 || ldw % 8 || ((reinterpret_cast<uintptr_t>(V) | reinterpret_cast<uintptr_t>(Vw)) & 15))
     return cudaErrorInvalidValue;
-  const int64_t total = N * (d / 8);
+  const int64_t d8 = (d + 7) / 8;
+  const int64_t total = N * d8;
   if (total == 0) return cudaSuccess;
   const int64_t blocks = std::min<int64_t>((total + 255) / 256, (int64_t)num_sms() * 8);
-  k_scale_rows<<<(unsigned)blocks, 256, 0, s>>>(V, ld, N, d / 8, w, Vw, ldw);
+  k_scale_rows<<<(unsigned)blocks, 256, 0, s>>>(V, ld, N, d8, w, Vw, ldw);
   note_launches(1);
   return cudaGetLastError();
 }

@@ -154,6 +154,8 @@ FIT_CASES = {
     # heavy-tailed inputs, n > m
     "student_small": synth.WORKLOADS["llama3_8b_down_14336x4096"].with_(N=20000, n=448, m=128,
                                                                         iters=4),
+    # fp32 samples whose widths are not multiples of 8 (padded bf16 rows on the tensor path)
+    "odd_f32": synth.WORKLOADS["tiny_64"].with_(N=3000, n=36, m=20, iters=5),
 }
 
 
