@@ -69,6 +69,17 @@ def measured_peaks():
             "fallback"
 
 
+def gram_source_sha256() -> str:
+    """sha256 of the Gram kernel's source: kernels_tc.cu from `namespace gram {` up to the
+    scaling pass that follows the Gram launcher (kernel, tile tables, reduction, launch)."""
+    src = os.path.join(ROOT, "paper_2609_14706_gb300", "csrc", "kernels_tc.cu")
+    with open(src) as f:
+        text = f.read()
+    a = text.index("namespace gram {")
+    b = text.index("__global__ void k_scale_rows")
+    return hashlib.sha256(text[a:b].encode()).hexdigest()
+
+
 def profiled_traffic(workload: str):
     """DRAM bytes per launch of the Gram kernel from the committed ncu summary, if the
     kernel source is still the one that was profiled (else None)."""
@@ -81,10 +92,8 @@ def profiled_traffic(workload: str):
     m2 = re.search(r"traffic_bytes_per_launch:\s*(\d+)", text)
     if not (m1 and m2):
         return None
-    src = os.path.join(ROOT, "paper_2609_14706_gb300", "csrc", "kernels_tc.cu")
-    with open(src, "rb") as f:
-        if hashlib.sha256(f.read()).hexdigest() != m1.group(1):
-            return None
+    if gram_source_sha256() != m1.group(1):
+        return None
     return int(m2.group(1))
 
 
