@@ -62,6 +62,31 @@ long long launches_so_far();
 constexpr int kGramBM = 256;
 constexpr int kGramBN = 256;
 constexpr int kGramBK = 64;   // samples per pipeline stage (weights padded to this)
+// The Gram tile table: the tiles that meet the lower triangle, listed by square supertiles
+// of kGramSuper x kGramSuper tiles (row-major over the supertiles of the lower triangle,
+// row-major inside each).  The persistent CTAs take consecutive units, so one wave of CTAs
+// covers about one supertile: its tiles share few operand feature blocks, which the CTAs
+// stream through L2 at about the same sample position.  lut[ti * nbn + tj] = the tile's
+// index, or -1 for tiles above the triangle.  Returns the tile count.
+constexpr int kGramSuper = 12;
+__host__ __device__ inline int gram_fill_tiles(int nbm, int nbn, int2* tiles, int* lut) {
+  int T = 0;
+  for (int I = 0; I < nbm; I += kGramSuper)
+    for (int J = 0; J < nbn && J <= I + kGramSuper - 1; J += kGramSuper)
+      for (int ti = I; ti < nbm && ti < I + kGramSuper; ++ti)
+        for (int tj = J; tj < nbn && tj < J + kGramSuper; ++tj) {
+          // tile meets the lower triangle iff its first column <= its last row
+          const bool need = (int64_t)tj * kGramBN <= (int64_t)ti * kGramBM + kGramBM - 1;
+          if (need) {
+            lut[ti * nbn + tj] = T;
+            tiles[T++] = make_int2(ti, tj);
+          }
+        }
+  for (int ti = 0; ti < nbm; ++ti)
+    for (int tj = 0; tj < nbn; ++tj)
+      if (!((int64_t)tj * kGramBN <= (int64_t)ti * kGramBM + kGramBM - 1)) lut[ti * nbn + tj] = -1;
+  return T;
+}
 struct GramPlan {
   int T;        // lower-triangle output tiles
   int S;        // K splits

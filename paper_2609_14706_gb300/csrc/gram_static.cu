@@ -47,13 +47,7 @@ void set_msg(char* buf, int32_t len, const char* msg) {
 __global__ void k_static_tiles(int64_t d, int nbm, int nbn, int2* tiles, int* lut) {
   // one thread: the tables are at most a few thousand entries
   if (blockIdx.x != 0 || threadIdx.x != 0) return;
-  int T = 0;
-  for (int ti = 0; ti < nbm; ++ti)
-    for (int tj = 0; tj < nbn; ++tj) {
-      const bool need = (int64_t)tj * kGramBN <= (int64_t)ti * kGramBM + kGramBM - 1;
-      lut[ti * nbn + tj] = need ? T : -1;
-      if (need) tiles[T++] = make_int2(ti, tj);
-    }
+  gram_fill_tiles(nbm, nbn, tiles, lut);
 }
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }

@@ -363,15 +363,7 @@ size_t gram_tile_table_bytes(int64_t d) {
 void gram_build_tiles(int64_t d, int2* tiles, int* lut, int* T_out) {
   const int nbm = (int)((d + gram::BM - 1) / gram::BM);
   const int nbn = (int)((d + gram::BN - 1) / gram::BN);
-  int T = 0;
-  for (int ti = 0; ti < nbm; ++ti)
-    for (int tj = 0; tj < nbn; ++tj) {
-      // tile meets the lower triangle iff its first column <= its last row
-      const bool need = (int64_t)tj * gram::BN <= (int64_t)ti * gram::BM + gram::BM - 1;
-      lut[ti * nbn + tj] = need ? T : -1;
-      if (need) tiles[T++] = make_int2(ti, tj);
-    }
-  *T_out = T;
+  *T_out = gram_fill_tiles(nbm, nbn, tiles, lut);
 }
 
 GramPlan gram_plan(int64_t N, int64_t d, int sms) {
