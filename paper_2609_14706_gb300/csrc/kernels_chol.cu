@@ -466,6 +466,266 @@ static cudaError_t gemm_tc(const Split& A, const Split& B, int nseg, const int a
 }
 
 // ---------------------------------------------------------------------------
+// Persistent trailing update C -= A' A'^T over the lower 128 x 128 tiles of an M x M block
+// (the columns beyond the next column block, on the side stream).  Each CTA walks its tiles
+// (t = blockIdx.x, + gridDim.x, ...) through one pipeline: the producer streams A' rows of
+// the tile's row and column blocks, the MMA issuer alternates two 128-column TMEM
+// accumulators, and the four epilogue warps drain tile j (C = alpha acc + beta C through
+// swizzled shared memory and TMA stores, each warp its 32 rows) while tile j+1's MMAs run.
+// Each epilogue warp loads its rows of the next tile's C as soon as its stores have read
+// the staging buffer.  C must be TMA-addressable (16-byte aligned rows).
+// ---------------------------------------------------------------------------
+namespace sy {
+constexpr int BM = 128, BN = 128, BK = 64, STAGES = 4;
+constexpr int A_BYTES = BM * BK * 2, B_BYTES = BN * BK * 2;
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int BOX = 32 * 128;           // 32 rows x 128 bytes (32 fp32)
+constexpr int WARP_C = 4 * BOX;         // an epilogue warp's 32 rows x 128 columns
+constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 4 * WARP_C + 256;
+constexpr uint32_t TMEM_COLS = 256;     // two 128-column accumulators
+}  // namespace sy
+
+struct SyrkArgs {
+  int ntiles;               // lower tiles: ntm (ntm + 1) / 2 for ntm = ceil(M / 128)
+  int nseg, kseg_blocks;    // K segments, 64-blocks per segment
+  int a_off[3], b_off[3];   // x offsets of the segments for the row / column operand
+  float alpha, beta;
+  DevStatus* st;
+};
+
+// tile t of the row-major lower triangle: t = tm (tm + 1) / 2 + tn, tn <= tm
+__device__ __forceinline__ void syrk_tile(int t, int& tm, int& tn) {
+  int r = (int)((sqrtf(8.f * (float)t + 1.f) - 1.f) * 0.5f);
+  while ((r + 1) * (r + 2) / 2 <= t) ++r;
+  while (r * (r + 1) / 2 > t) --r;
+  tm = r;
+  tn = t - r * (r + 1) / 2;
+}
+
+__global__ void __launch_bounds__(256, 1)
+    k_syrk_tc(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap cmap,
+              const SyrkArgs a) {
+  using namespace sy;
+  pdl_enter();
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint8_t* cst = smem + STAGES * STAGE_BYTES;  // [epilogue warp][4 boxes]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(cst + 4 * WARP_C);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + STAGES;
+  uint64_t* accf = bars + 2 * STAGES;  // [2]
+  uint64_t* acce = accf + 2;           // [2]
+  uint64_t* cbar = acce + 2;           // [4]
+  uint64_t* drain = cbar + 4;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  volatile int* skip_flag = abort_flag + 1;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    *skip_flag = *reinterpret_cast<volatile int*>(&a.st->abort_all);
+    *abort_flag = 0;
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&accf[b], 1);
+      mbar_init(&acce[b], 4);
+    }
+    for (int w = 0; w < 4; ++w) mbar_init(&cbar[w], 1);
+    mbar_init(drain, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (*skip_flag) return;
+  const int wq = warp - 4;
+  if (warp >= 4 && lane == 0 && (int)blockIdx.x < a.ntiles) {
+    // the first tile's C rows of this epilogue warp
+    int tm, tn;
+    syrk_tile(blockIdx.x, tm, tn);
+    mbar_arrive_expect_tx(&cbar[wq], WARP_C);
+    for (int cb = 0; cb < 4; ++cb)
+      tma_load_3d(cst + wq * WARP_C + cb * BOX, &cmap, &cbar[wq], tn * BN + 32 * cb,
+                  tm * BM + 32 * wq, 0);
+  }
+  if (warp == 2) {
+    tmem_alloc(tmem_slot, TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const int nk = a.nseg * a.kseg_blocks;
+
+  if (warp == 0 && lane == 0) {
+    bool ok = true;
+    int it = 0;
+    for (int t = blockIdx.x; t < a.ntiles && ok; t += gridDim.x) {
+      int tm, tn;
+      syrk_tile(t, tm, tn);
+      for (int i = 0; i < nk; ++i, ++it) {
+        const int s = it % STAGES;
+        const uint32_t ph = (it / STAGES) & 1;
+        if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, kGemmWaitNs)) {
+          ok = false;
+          break;
+        }
+        const int seg = i / a.kseg_blocks, kb = i - seg * a.kseg_blocks;
+        mbar_arrive_expect_tx(&full[s], STAGE_BYTES);
+        uint8_t* sa = smem + s * STAGE_BYTES;
+        tma_load_2d(sa, &amap, &full[s], a.a_off[seg] + kb * BK, tm * BM);
+        tma_load_2d(sa + A_BYTES, &amap, &full[s], a.b_off[seg] + kb * BK, tn * BN);
+      }
+    }
+    if (!ok) {
+      *abort_flag = 1;
+      raise_error(a.st, FFH_ERR_TIMEOUT, 25);
+    }
+    const int first = it > STAGES ? it - STAGES : 0;
+    for (int j = first; j < it; ++j) {
+      volatile int never = 0;
+      mbar_wait(&full[j % STAGES], (j / STAGES) & 1, &never, kGemmWaitNs);
+    }
+  } else if (warp == 1 && lane == 0) {
+    constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, false, false);
+    bool ok = true;
+    int it = 0, j = 0;
+    for (int t = blockIdx.x; t < a.ntiles && ok; t += gridDim.x, ++j) {
+      const int buf = j & 1;
+      if (!mbar_wait(&acce[buf], ((j >> 1) & 1) ^ 1, abort_flag, kGemmWaitNs)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      for (int i = 0; i < nk; ++i, ++it) {
+        const int s = it % STAGES;
+        const uint32_t ph = (it / STAGES) & 1;
+        if (!mbar_wait(&full[s], ph, abort_flag, kGemmWaitNs)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t sa = smem_u32(smem + s * STAGE_BYTES), sb = sa + A_BYTES;
+#pragma unroll
+        for (int k = 0; k < BK / 16; ++k)
+          mma_bf16(tmem + buf * BN, sw128_desc(sa + k * 32, 16, 1024),
+                   sw128_desc(sb + k * 32, 16, 1024), idesc, (i > 0 || k > 0) ? 1u : 0u);
+        mma_commit(&empty[s]);
+      }
+      if (!ok) break;
+      mma_commit(&accf[buf]);
+    }
+    if (!ok) {
+      *abort_flag = 1;
+      raise_error(a.st, FFH_ERR_TIMEOUT, 26);
+    }
+    mma_commit(drain);
+    volatile int never = 0;
+    mbar_wait(drain, 0, &never, kGemmWaitNs);
+  } else if (warp >= 4) {
+    uint8_t* wc = cst + wq * WARP_C;
+    int j = 0;
+    for (int t = blockIdx.x; t < a.ntiles; t += gridDim.x, ++j) {
+      const int buf = j & 1;
+      int tm, tn;
+      syrk_tile(t, tm, tn);
+      bool ok = mbar_wait(&cbar[wq], j & 1, abort_flag, kGemmWaitNs);
+      if (ok) ok = mbar_wait(&accf[buf], (j >> 1) & 1, abort_flag, kGemmWaitNs);
+      if (!ok) {
+        if (lane == 0) {
+          *abort_flag = 1;
+          raise_error(a.st, FFH_ERR_TIMEOUT, 27);
+        }
+        break;
+      }
+      tc_fence_after();
+#pragma unroll 1
+      for (int cb = 0; cb < 4; ++cb) {
+        float v[32];
+        tmem_ld32(tmem + ((uint32_t)(wq * 32) << 16) + buf * BN + cb * 32, v);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          float4* cp = reinterpret_cast<float4*>(wc + cb * BOX + sw128_off(lane, q));
+          const float4 pv = *cp;
+          *cp = make_float4(fmaf(a.beta, pv.x, a.alpha * v[4 * q]),
+                            fmaf(a.beta, pv.y, a.alpha * v[4 * q + 1]),
+                            fmaf(a.beta, pv.z, a.alpha * v[4 * q + 2]),
+                            fmaf(a.beta, pv.w, a.alpha * v[4 * q + 3]));
+        }
+      }
+      // this warp's reads of the accumulator are done
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acce[buf]);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        for (int cb = 0; cb < 4; ++cb)
+          tma_store_3d(&cmap, wc + cb * BOX, tn * BN + 32 * cb, tm * BM + 32 * wq, 0);
+        bulk_commit_group();
+        bulk_wait_read_all();
+        const int tnext = t + gridDim.x;
+        if (tnext < a.ntiles) {
+          int tm2, tn2;
+          syrk_tile(tnext, tm2, tn2);
+          mbar_arrive_expect_tx(&cbar[wq], WARP_C);
+          for (int cb = 0; cb < 4; ++cb)
+            tma_load_3d(wc + cb * BOX, &cmap, &cbar[wq], tn2 * BN + 32 * cb, tm2 * BM + 32 * wq,
+                        0);
+        }
+      }
+      __syncwarp();
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+// C (M x M, pitch ldc) -= A' A'^T on the lower tiles, A' = the split rows of A.  Returns
+// cudaErrorNotSupported when C's layout is not TMA-addressable (the caller then uses
+// gemm_tc).  grid_cap bounds the persistent CTAs (SMs left to the other stream).
+static cudaError_t syrk_tc(const Split& A, const int a_seg[3], const int b_seg[3], int nseg,
+                           int kseg, float* C, int64_t ldc, int M, float alpha, float beta,
+                           int grid_cap, DevStatus* st, cudaStream_t s) {
+  if (M <= 0) return cudaSuccess;
+  CUtensorMap am, cm;
+  if (!map_epi_3d(&cm, C, false, (uint64_t)M, (uint64_t)M, 1, (uint64_t)ldc, 0))
+    return cudaErrorNotSupported;
+  if (!map_bf16_kmajor(&am, A.p, (uint64_t)2 * A.kpad, (uint64_t)A.rows_pad * A.batch,
+                       (uint64_t)2 * A.kpad, sy::BM))
+    return cudaErrorInvalidValue;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k_syrk_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         sy::SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  SyrkArgs g{};
+  const int ntm = (M + sy::BM - 1) / sy::BM;
+  g.ntiles = ntm * (ntm + 1) / 2;
+  g.nseg = nseg;
+  g.kseg_blocks = (kseg + sy::BK - 1) / sy::BK;
+  for (int i = 0; i < 3; ++i) {
+    g.a_off[i] = a_seg[i];
+    g.b_off[i] = b_seg[i];
+  }
+  g.alpha = alpha;
+  g.beta = beta;
+  g.st = st;
+  const int grid = std::max(1, std::min(g.ntiles, grid_cap));
+  cudaError_t e = launch_pdl(k_syrk_tc, dim3(grid), dim3(256), sy::SMEM_BYTES, s, am, cm, g);
+  note_launches(1);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
 // fp32 -> bf16 hi/lo split, optionally transposed, batched:
 //   batch z, row r < rows, col c < cols of the source view
 //     src[z*src_stride + r*lds + c]          (trans = 0)
@@ -1075,9 +1335,15 @@ static cudaError_t cholesky_tc_body(const float* F, int64_t d, int64_t ldf, floa
     if ((e = cudaStreamWaitEvent(cs->side, cs->ev[1], 0)) != cudaSuccess) return e;
     if (rows > LB) {
       Split rest{l21.p + (size_t)LB * 2 * l21.kpad, rows_pad - LB, 128, 1};
-      if ((e = gemm_tc(rest, rest, 3, aseg, bseg, 128, W + (o + 2 * LB) * d + (o + 2 * LB), d, 0,
-                       rows - LB, rows - LB, -1.f, 1.f, true, 1, st, cs->side)) != cudaSuccess)
-        return e;
+      float* C22 = W + (o + 2 * LB) * d + (o + 2 * LB);
+      // persistent, leaving SMs to the critical stream's kernels (each uses at most
+      // d / 128 CTAs, one at a time)
+      const int cap = num_sms() - (int)std::min<int64_t>((d + 127) / 128 + 8, num_sms() / 2);
+      e = syrk_tc(rest, aseg, bseg, 3, 128, C22, d, rows - LB, -1.f, 1.f, cap, st, cs->side);
+      if (e == cudaErrorNotSupported)
+        e = gemm_tc(rest, rest, 3, aseg, bseg, 128, C22, d, 0, rows - LB, rows - LB, -1.f, 1.f,
+                    true, 1, st, cs->side);
+      if (e != cudaSuccess) return e;
     }
     if ((e = cudaEventRecord(cs->ev[2 + (p & 1)], cs->side)) != cudaSuccess) return e;
     // critical: the next column block, A22[:, :128] -= L21 L21[:128]^T, after the side
