@@ -1336,9 +1336,9 @@ static cudaError_t cholesky_tc_body(const float* F, int64_t d, int64_t ldf, floa
     if (rows > LB) {
       Split rest{l21.p + (size_t)LB * 2 * l21.kpad, rows_pad - LB, 128, 1};
       float* C22 = W + (o + 2 * LB) * d + (o + 2 * LB);
-      // persistent, leaving SMs to the critical stream's kernels (each uses at most
-      // d / 128 CTAs, one at a time)
-      const int cap = num_sms() - (int)std::min<int64_t>((d + 127) / 128 + 8, num_sms() / 2);
+      // persistent, leaving 24 SMs to the critical stream's kernels (at large d this update
+      // is the bottleneck: reserving d / 128 + 8 SMs, or 48, measured slower)
+      const int cap = num_sms() - 24;
       e = syrk_tc(rest, aseg, bseg, 3, 128, C22, d, rows - LB, -1.f, 1.f, cap, st, cs->side);
       if (e == cudaErrorNotSupported)
         e = gemm_tc(rest, rest, 3, aseg, bseg, 128, C22, d, 0, rows - LB, rows - LB, -1.f, 1.f,
