@@ -5,8 +5,9 @@
 //   * k_chol_leaf  factors the 128 x 128 diagonal block in shared memory (one CTA) and,
 //                  in the same column sweep, its inverse M11 = L11^-1 (each elimination
 //                  step applied to the identity as well);
-//   * the panel below, L21 = A21 M11^T, and the trailing update A22 -= L21 L21^T are
-//     tcgen05 GEMMs (k_gemm_tc);
+//   * the panel below, L21 = A21 M11^T, and the trailing update of the next column
+//     block are tcgen05 GEMMs (k_gemm_tc); the trailing update A22 -= L21 L21^T of the
+//     columns beyond it is a persistent tcgen05 kernel on a side stream (k_syrk_tc);
 // then M = L^-1 by recursive doubling over the diagonal-block inverses:
 //   [[L11, 0], [L21, L22]]^-1 = [[M11, 0], [-M22 (L21 M11), M22]].
 //
