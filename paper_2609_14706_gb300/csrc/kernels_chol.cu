@@ -321,6 +321,12 @@ __global__ void __launch_bounds__(256, 1)
     } else if (lane == 0) {
       *abort_flag = 1;
       raise_error(a.st, FFH_ERR_TIMEOUT, 23);
+      // this warp's beta-C copy may still be in flight: let it land (bounded) before the
+      // CTA's shared memory is released
+      if (load_c) {
+        volatile int never = 0;
+        mbar_wait(&cbar[warp], 0, &never, kGemmWaitNs);
+      }
     }
   } else if (warp >= 4) {
     if (mbar_wait(accf, 0, abort_flag, kGemmWaitNs)) {
@@ -638,6 +644,10 @@ __global__ void __launch_bounds__(256, 1)
         if (lane == 0) {
           *abort_flag = 1;
           raise_error(a.st, FFH_ERR_TIMEOUT, 27);
+          // this tile's C copy may still be in flight: let it land (bounded) before the
+          // CTA's shared memory is released
+          volatile int never = 0;
+          mbar_wait(&cbar[wq], j & 1, &never, kGemmWaitNs);
         }
         break;
       }
