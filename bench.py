@@ -225,6 +225,25 @@ def run_reference(args):
 
 
 # ---------------------------------------------------------------------------
+# multi-rank aggregation (independent fits, one per rank)
+# ---------------------------------------------------------------------------
+def max_over_ranks(value: float, dist, device) -> float:
+    """The largest `value` over all ranks, returned on every rank: the job takes as long
+    as its slowest rank."""
+    if dist is None:
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world: int, steps: int, iters_per_step: int, elapsed_ms: float) -> float:
+    """Iterations per second of the whole job: each of the `world` ranks fits its own layer,
+    so world x steps x iters iterations complete in the slowest rank's time."""
+    return world * steps * iters_per_step / (elapsed_ms / 1e3)
+
+
+# ---------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------
 def run_ours(args):
@@ -288,11 +307,8 @@ def run_ours(args):
     elapsed_ms = e0.elapsed_time(e1)
     tim = h.timings()
     launches = tim["kernel_launches"] - launches0
-    if dist is not None:
-        t = torch.tensor([elapsed_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
-    value = world * args.steps * iters / (elapsed_ms / 1e3)
+    elapsed_ms = max_over_ranks(elapsed_ms, dist, "cuda")
+    value = whole_job_rate(world, args.steps, iters, elapsed_ms)
 
     # ---- end to end through the C ABI with host buffers
     e2e = None
@@ -313,13 +329,9 @@ def run_ours(args):
         f1.record(stream)
         barrier()
         wall_ms = (time.perf_counter() - t0) * 1e3
-        e2e_ms = max(f0.elapsed_time(f1), wall_ms)
-        if dist is not None:
-            t = torch.tensor([e2e_ms], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_ms = float(t.item())
+        e2e_ms = max_over_ranks(max(f0.elapsed_time(f1), wall_ms), dist, "cuda")
         h2.close()
-        e2e = {"value": world * args.steps * iters / (e2e_ms / 1e3), "unit": UNIT,
+        e2e = {"value": whole_job_rate(world, args.steps, iters, e2e_ms), "unit": UNIT,
                "h2d_bytes_per_step": Xh.numel() * Xh.element_size() + Gh.numel() * Gh.element_size(),
                "d2h_bytes_per_step": (n * n + m * m) * 4}
         del Xh, Gh
