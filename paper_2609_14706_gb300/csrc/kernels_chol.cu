@@ -806,8 +806,8 @@ static cudaError_t split(const float* src, int64_t lds, int64_t src_stride, int 
 //   A(q)  warp 0 factors the 32 x 32 diagonal block D_q and inverts it in registers:
 //         lane i holds row i of D_q and column i of its inverse; the 2 x 2 pivot block
 //         of columns j, j+1 is broadcast by shuffle, and the remaining columns shift
-//         down two registers per step so every register index is static.  Writes L_qq, Mi_q = L_qq^-1 and
-//         Mt[x][k] = Mi_q[k][x].
+//         down two registers per step so every register index is static.  Writes L_qq,
+//         Mi_q = L_qq^-1 and Mt[x][k] = Mi_q[k][x].
 //   B(q)  all warps: the rows below, L[r][Q] = A[r][Q] Mi_q^T (4 x 4 register blocks),
 //         also stored transposed, Pt[k][r] = L[r][32q+k].
 //   C(q)  warps 0-1 apply the rank-32 update of sub-panel q to D_{q+1} and warp 0 goes
