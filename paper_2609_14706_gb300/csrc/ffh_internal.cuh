@@ -69,6 +69,15 @@ constexpr int kGramBK = 64;   // samples per pipeline stage (weights padded to t
 // stream through L2 at about the same sample position.  lut[ti * nbn + tj] = the tile's
 // index, or -1 for tiles above the triangle.  Returns the tile count.
 constexpr int kGramSuper = 12;
+// Tile t of a row-major lower triangle of tiles: t = tm (tm + 1) / 2 + tn with tn <= tm (the
+// float square root gives a first guess, the integer steps make it exact).
+__host__ __device__ inline void lower_tile(int t, int& tm, int& tn) {
+  int r = (int)((sqrtf(8.f * (float)t + 1.f) - 1.f) * 0.5f);
+  while ((r + 1) * (r + 2) / 2 <= t) ++r;
+  while (r * (r + 1) / 2 > t) --r;
+  tm = r;
+  tn = t - r * (r + 1) / 2;
+}
 __host__ __device__ inline int gram_fill_tiles(int nbm, int nbn, int2* tiles, int* lut) {
   int T = 0;
   for (int I = 0; I < nbm; I += kGramSuper)

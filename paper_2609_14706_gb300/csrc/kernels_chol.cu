@@ -500,15 +500,6 @@ struct SyrkArgs {
   DevStatus* st;
 };
 
-// tile t of the row-major lower triangle: t = tm (tm + 1) / 2 + tn, tn <= tm
-__device__ __forceinline__ void syrk_tile(int t, int& tm, int& tn) {
-  int r = (int)((sqrtf(8.f * (float)t + 1.f) - 1.f) * 0.5f);
-  while ((r + 1) * (r + 2) / 2 <= t) ++r;
-  while (r * (r + 1) / 2 > t) --r;
-  tm = r;
-  tn = t - r * (r + 1) / 2;
-}
-
 __global__ void __launch_bounds__(256, 1)
     k_syrk_tc(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap cmap,
               const SyrkArgs a) {
@@ -550,7 +541,7 @@ __global__ void __launch_bounds__(256, 1)
   if (warp >= 4 && lane == 0 && (int)blockIdx.x < a.ntiles) {
     // the first tile's C rows of this epilogue warp
     int tm, tn;
-    syrk_tile(blockIdx.x, tm, tn);
+    lower_tile(blockIdx.x, tm, tn);
     mbar_arrive_expect_tx(&cbar[wq], WARP_C);
     for (int cb = 0; cb < 4; ++cb)
       tma_load_3d(cst + wq * WARP_C + cb * BOX, &cmap, &cbar[wq], tn * BN + 32 * cb,
@@ -571,7 +562,7 @@ __global__ void __launch_bounds__(256, 1)
     int it = 0;
     for (int t = blockIdx.x; t < a.ntiles && ok; t += gridDim.x) {
       int tm, tn;
-      syrk_tile(t, tm, tn);
+      lower_tile(t, tm, tn);
       for (int i = 0; i < nk; ++i, ++it) {
         const int s = it % STAGES;
         const uint32_t ph = (it / STAGES) & 1;
@@ -637,7 +628,7 @@ __global__ void __launch_bounds__(256, 1)
     for (int t = blockIdx.x; t < a.ntiles; t += gridDim.x, ++j) {
       const int buf = j & 1;
       int tm, tn;
-      syrk_tile(t, tm, tn);
+      lower_tile(t, tm, tn);
       bool ok = mbar_wait(&cbar[wq], j & 1, abort_flag, kGemmWaitNs);
       if (ok) ok = mbar_wait(&accf[buf], (j >> 1) & 1, abort_flag, kGemmWaitNs);
       if (!ok) {
@@ -680,7 +671,7 @@ __global__ void __launch_bounds__(256, 1)
         const int tnext = t + gridDim.x;
         if (tnext < a.ntiles) {
           int tm2, tn2;
-          syrk_tile(tnext, tm2, tn2);
+          lower_tile(tnext, tm2, tn2);
           mbar_arrive_expect_tx(&cbar[wq], WARP_C);
           for (int cb = 0; cb < 4; ++cb)
             tma_load_3d(wc + cb * BOX, &cmap, &cbar[wq], tn2 * BN + 32 * cb, tm2 * BM + 32 * wq,

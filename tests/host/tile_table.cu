@@ -1,7 +1,8 @@
-// Host-only check of the Gram tile table (gram_fill_tiles): every 256 x 256 output tile that
-// meets the lower triangle is listed exactly once, the lookup table maps each listed tile to
-// its index and every other tile to -1, and consecutive entries stay inside square
-// supertiles.  Prints "ok" or the first violation; exit status 0 on success.
+// Host-only checks of the tile bookkeeping: the Gram tile table (gram_fill_tiles) lists every
+// 256 x 256 output tile that meets the lower triangle exactly once, its lookup table maps
+// each listed tile to its index and every other tile to -1, and consecutive entries stay
+// inside square supertiles; lower_tile (the persistent Cholesky update's tile walk) maps
+// 0..T-1 onto the lower triangle in row-major order.  Prints "ok" or the first violation.
 #include <cstdio>
 #include <vector>
 
@@ -40,9 +41,24 @@ static int check(int64_t d) {
   return 0;
 }
 
+// lower_tile: a bijection from 0..T-1 onto the tiles (tm, tn), tn <= tm, in row-major order
+static int check_lower_tile(int ntm) {
+  int t = 0;
+  for (int tm = 0; tm < ntm; ++tm)
+    for (int tn = 0; tn <= tm; ++tn, ++t) {
+      int a, b;
+      lower_tile(t, a, b);
+      if (a != tm || b != tn)
+        return printf("lower_tile(%d) = (%d,%d), expected (%d,%d)\n", t, a, b, tm, tn), 1;
+    }
+  return 0;
+}
+
 int main() {
   for (int64_t d : {1, 64, 255, 256, 257, 4096, 3000, 11008, 14336, 40000})
     if (check(d)) return 1;
+  // up to a 65536 x 65536 trailing matrix of 128 x 128 tiles
+  if (check_lower_tile(512)) return 1;
   printf("ok\n");
   return 0;
 }

@@ -1,6 +1,7 @@
 """Host-side logic of the library checked on the CPU (no GPU): the Gram tile table that
-the persistent Gram kernel and its reduction share (tests/host/tile_table.cu, compiled with
-nvcc as a host-only program)."""
+the persistent Gram kernel and its reduction share, and the lower-triangle tile walk of the
+persistent Cholesky update (tests/host/tile_table.cu, compiled with nvcc as a host-only
+program)."""
 import os
 import shutil
 import subprocess
