@@ -30,7 +30,11 @@ Readings where the paper is silent (each also listed in the design notes):
     notation) and forward substitution: v^T F^-1 v = ||L^-1 v||^2.
 
 All arithmetic is fp64 numpy/scipy; LAPACK's Cholesky, triangular solve and BLAS
-matmul are used as library primitives, with no blocking or fusion of our own.
+matmul are used as library primitives.  The only grouping of our own is that the sums
+over the N samples (the empirical expectations) are accumulated over consecutive
+blocks of rows, so that samples stored in a narrow type (bf16) are widened to fp64 one
+block at a time and the full-size workloads fit in host memory; the sum and its terms
+are unchanged, only the order of the additions.
 """
 from __future__ import annotations
 
@@ -80,6 +84,46 @@ def inv_quad_forms_chol(L: np.ndarray, V: np.ndarray) -> np.ndarray:
     return np.einsum("ik,ik->k", Y, Y)
 
 
+# rows widened to fp64 at a time by the fits (a block of 16384 rows of 14336 features
+# is 1.9 GB)
+BLOCK_ROWS = 16384
+
+
+def row_blocks(V, rows: int = BLOCK_ROWS):
+    """Yield (r0, r1, fp64 copy of rows r0..r1-1) of V (numpy array or torch tensor of
+    any float dtype)."""
+    N = V.shape[0]
+    for r0 in range(0, N, rows):
+        r1 = min(N, r0 + rows)
+        yield r0, r1, as_f64(V[r0:r1])
+
+
+def inv_quad_forms_rows(L: np.ndarray, V, rows: int = BLOCK_ROWS) -> np.ndarray:
+    """inv_quad_forms_chol over all rows of V, a block of rows at a time."""
+    q = np.empty(V.shape[0])
+    for r0, r1, Vb in row_blocks(V, rows):
+        q[r0:r1] = inv_quad_forms_chol(L, Vb)
+    return q
+
+
+def sq_norms_rows(V, rows: int = BLOCK_ROWS) -> np.ndarray:
+    """||v_k||^2 = v_k^T I^-1 v_k for every row (the weights at A_0 = I)."""
+    q = np.empty(V.shape[0])
+    for r0, r1, Vb in row_blocks(V, rows):
+        q[r0:r1] = np.einsum("kd,kd->k", Vb, Vb)
+    return q
+
+
+def weighted_gram_rows(V, w: np.ndarray, scale: float, rows: int = BLOCK_ROWS) -> np.ndarray:
+    """scale * sum_k w_k v_k v_k^T (weighted_gram), the sum over k accumulated a block
+    of rows at a time."""
+    d = V.shape[1]
+    C = np.zeros((d, d))
+    for r0, r1, Vb in row_blocks(V, rows):
+        C += weighted_gram(Vb, w[r0:r1], 1.0)
+    return scale * C
+
+
 def fwd_quad_forms(F: np.ndarray, V: np.ndarray) -> np.ndarray:
     """q_k = v_k^T F v_k (the Frobenius variant's weights, Section 5)."""
     return np.einsum("kd,kd->k", V @ F, V)
@@ -87,7 +131,13 @@ def fwd_quad_forms(F: np.ndarray, V: np.ndarray) -> np.ndarray:
 
 def weighted_gram(V: np.ndarray, w: np.ndarray, scale: float) -> np.ndarray:
     """scale * sum_k w_k v_k v_k^T = scale * V^T diag(w) V (Section 5: the
-    expectations E[(.) x x^T] and E[(.) g g^T] as empirical means)."""
+    expectations E[(.) x x^T] and E[(.) g g^T] as empirical means).  With all w_k >= 0
+    (the flip-flop weights are quadratic forms of SPD matrices) each term is written
+    (sqrt(w_k) v_k)(sqrt(w_k) v_k)^T, so the product is a symmetric rank-k update."""
+    w = np.asarray(w, dtype=np.float64)
+    if np.all(w >= 0.0):
+        Vs = V * np.sqrt(w)[:, None]
+        return scale * (Vs.T @ Vs)
     return scale * ((V.T * w) @ V)
 
 
@@ -157,43 +207,51 @@ class FitResult:
     mean_qr: List[float]
     q: Optional[np.ndarray] = None   # last q (x^T A^-1 x with the returned A)
     r: Optional[np.ndarray] = None   # last r (g^T B^-1 g with the returned B)
+    # (A_t, B_t) after every iteration, when asked for
+    iterates: List = dataclasses.field(default_factory=list)
 
 
 def flipflop_fit(X, G, iters: int, tol: float = 0.0, damping: float = 0.0,
-                 init_A=None) -> FitResult:
+                 init_A=None, rows: int = BLOCK_ROWS, keep_iterates: bool = False,
+                 progress=None) -> FitResult:
     """FlipFlop Hessian fit of A (n x n) and B (m x m) to rank-one samples.
 
-    X: N x n (rows x_k^T), G: N x m (rows g_k^T).  Section 5 flip-flop updates with
-    the Appendix B settings (A_0 = I_n unless init_A is given; iteration = B-update,
-    then A-update), MLE constants, tr(A) = n normalisation after each iteration.
+    X: N x n (rows x_k^T), G: N x m (rows g_k^T), numpy arrays or host torch tensors
+    of any float dtype (widened to fp64 a block of `rows` rows at a time).  Section 5
+    flip-flop updates with the Appendix B settings (A_0 = I_n unless init_A is given;
+    iteration = B-update, then A-update), MLE constants, tr(A) = n normalisation after
+    each iteration.  keep_iterates: also return every (A_t, B_t).  progress: called
+    with (t, delta_t) after each iteration.
     """
-    X, G = as_f64(X), as_f64(G)
+    if not hasattr(X, "shape") or not hasattr(G, "shape"):
+        X, G = as_f64(X), as_f64(G)
     N, n = X.shape
     m = G.shape[1]
     if init_A is None:
         A = np.eye(n)
-        q = np.einsum("kd,kd->k", X, X)           # x^T I^-1 x
+        q = sq_norms_rows(X, rows)                # x^T I^-1 x
         logdet_A = 0.0
     else:
         A = as_f64(init_A)
         LA = cholesky(A)
-        q = inv_quad_forms_chol(LA, X)
+        q = inv_quad_forms_rows(LA, X, rows)
         logdet_A = logdet_from_cholesky(LA)
     B_prev = None
     A_prev = A.copy()
     deltas, lls, mqr = [], [], []
+    iterates = []
     t_done = 0
     r = None
     for t in range(1, iters + 1):
         # B-update with A fixed: B = 1/(N n) sum_k q_k g_k g_k^T
-        B = damp(weighted_gram(G, q, 1.0 / (N * n)), damping)
+        B = damp(weighted_gram_rows(G, q, 1.0 / (N * n), rows), damping)
         LB = cholesky(B)
         logdet_B = logdet_from_cholesky(LB)
-        r = inv_quad_forms_chol(LB, G)
+        r = inv_quad_forms_rows(LB, G, rows)
         lls.append(gaussian_loglik(N, n, m, logdet_A, logdet_B, float(np.dot(q, r))))
         mqr.append(float(np.mean(q * r)))
         # A-update with B fixed: A = 1/(N m) sum_k r_k x_k x_k^T
-        A = damp(weighted_gram(X, r, 1.0 / (N * m)), damping)
+        A = damp(weighted_gram_rows(X, r, 1.0 / (N * m), rows), damping)
         # scale freedom: tr(A) = n, B carries the scale
         s = np.trace(A) / n
         A = A / s
@@ -202,18 +260,22 @@ def flipflop_fit(X, G, iters: int, tol: float = 0.0, damping: float = 0.0,
         r = r / s
         LA = cholesky(A)
         logdet_A = logdet_from_cholesky(LA)
-        q = inv_quad_forms_chol(LA, X)
+        q = inv_quad_forms_rows(LA, X, rows)
         lls.append(gaussian_loglik(N, n, m, logdet_A, logdet_B, float(np.dot(q, r))))
         mqr.append(float(np.mean(q * r)))
         delta = math.inf if B_prev is None else max(rel_change(A, A_prev),
                                                     rel_change(B, B_prev))
         deltas.append(delta)
         A_prev, B_prev = A.copy(), B.copy()
+        if keep_iterates:
+            iterates.append((A_prev, B_prev))
         t_done = t
+        if progress is not None:
+            progress(t, delta)
         if tol > 0.0 and delta < tol:
             break
     return FitResult(A=A, B=B, iters_done=t_done, deltas=deltas, loglik=lls,
-                     mean_qr=mqr, q=q, r=r)
+                     mean_qr=mqr, q=q, r=r, iterates=iterates)
 
 
 def flipflop_fit_matrix(Gk, iters: int, tol: float = 0.0, damping: float = 0.0,

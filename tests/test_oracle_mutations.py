@@ -23,12 +23,18 @@ def _checks():
         "quad_vs_inverse": lambda: pins.test_quad_forms_vs_explicit_inverse(),
         "brute_force": lambda: pins.test_brute_force_minimiser_agrees(),
         "matrix_eq_rank1": lambda: pins.test_matrix_variant_equals_rank_one_variant(),
+        "delta_hand": lambda: pins.test_delta_hand_computed_2x2(),
+        "delta_invariance": lambda: pins.test_delta_invariant_under_kronecker_rescaling(),
+        "delta_iterates": lambda: pins.test_fit_delta_compares_consecutive_iterates(),
+        "damped_stationary":
+            lambda: pins.test_damped_fixed_point_satisfies_damped_stationary_equations(),
     }
 
 
 _orig_gram = ff.weighted_gram
 _orig_quad = ff.inv_quad_forms_chol
 _orig_fit = ff.flipflop_fit
+_orig_damp = ff.damp
 
 MUTATIONS = {
     # the weights q_k / r_k are dropped from the Gram
@@ -43,6 +49,15 @@ MUTATIONS = {
                               sla.solve_triangular(L.T, V.T, lower=True))),
     # q_k squared (an exponent slip)
     "squared_weight": ("inv_quad_forms_chol", lambda L, V: _orig_quad(L, V) ** 2),
+    # delta_t without the trace normalisation of either iterate
+    "delta_unnormalised": ("rel_change",
+                           lambda F, P: float(np.linalg.norm(F - P) / np.linalg.norm(F))),
+    # delta_t relative to the previous iterate instead of the new one
+    "delta_old_denominator": ("rel_change", lambda F, P: float(
+        np.linalg.norm(F / np.trace(F) - P / np.trace(P)) / np.linalg.norm(P / np.trace(P)))),
+    # the damping shift lambda tr(F) instead of lambda mean(diag F)
+    "damping_trace_not_mean": ("damp", lambda F, lam: F if lam == 0.0 else
+                               F + lam * float(np.trace(F)) * np.eye(F.shape[0])),
 }
 
 
@@ -92,3 +107,37 @@ def test_pins_catch_missing_normalisation(monkeypatch):
         except (AssertionError, np.linalg.LinAlgError, ValueError):
             failed.append(cname)
     assert failed
+
+
+def _run_checks():
+    failed = []
+    for cname, check in _checks().items():
+        try:
+            check()
+        except (AssertionError, np.linalg.LinAlgError, ValueError, FloatingPointError):
+            failed.append(cname)
+    return failed
+
+
+def test_pins_catch_damping_of_one_factor_only(monkeypatch):
+    """Appendix B damps both factors; damping only the B-updates (every other call)."""
+    calls = {"n": 0}
+
+    def one_sided(F, lam):
+        calls["n"] += 1
+        return _orig_damp(F, lam) if calls["n"] % 2 == 1 else F
+    monkeypatch.setattr(ff, "damp", one_sided)
+    monkeypatch.setattr(oracle, "damp", one_sided)
+    assert _run_checks()
+
+
+def test_pins_catch_damping_only_of_the_returned_pair(monkeypatch):
+    """Appendix B damps "including between iterations"; damping only the factors that
+    are returned (the iteration itself undamped)."""
+    def late(X, G, *a, damping=0.0, **k):
+        r = _orig_fit(X, G, *a, **k)
+        r.A, r.B = _orig_damp(r.A, damping), _orig_damp(r.B, damping)
+        return r
+    monkeypatch.setattr(ff, "flipflop_fit", late)
+    monkeypatch.setattr(oracle, "flipflop_fit", late)
+    assert _run_checks()

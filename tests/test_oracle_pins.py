@@ -232,6 +232,118 @@ def test_damping_breaks_trace_identity_as_expected():
     assert np.trace(f.B) != pytest.approx(np.trace(f1.B), rel=1e-6)
 
 
+def test_delta_hand_computed_2x2():
+    """delta_t's definition worked by hand: A_t = diag(2, 1), A_{t-1} = I_2 give
+    A^_t = diag(2/3, 1/3), A^_{t-1} = diag(1/2, 1/2), difference diag(1/6, -1/6) with
+    norm sqrt(2)/6, ||A^_t|| = sqrt(5)/3, so delta = 1/sqrt(10).  A missing trace
+    normalisation gives 1/sqrt(5), the norm of A^_{t-1} in the denominator 1/3."""
+    At = np.diag([2.0, 1.0])
+    Ap = np.eye(2)
+    assert oracle.rel_change(At, Ap) == pytest.approx(1.0 / math.sqrt(10.0), rel=1e-15)
+    # an off-diagonal pair: A_t = [[3, 1], [1, 1]] (tr 4), A_{t-1} = [[1, 0], [0, 3]]
+    # (tr 4): difference [[2, 1], [1, -2]] / 4, norm sqrt(10)/4; ||A^_t|| = sqrt(12)/4
+    At = np.array([[3.0, 1.0], [1.0, 1.0]])
+    Ap = np.array([[1.0, 0.0], [0.0, 3.0]])
+    assert oracle.rel_change(At, Ap) == pytest.approx(math.sqrt(10.0 / 12.0), rel=1e-15)
+
+
+def test_delta_invariant_under_kronecker_rescaling():
+    """The fixed point is defined only up to (c A, B / c) (Section 5), so delta must not
+    change when either iterate of either factor is rescaled."""
+    rng = np.random.default_rng(21)
+    for _ in range(5):
+        a = rng.standard_normal((4, 4))
+        b = rng.standard_normal((4, 4))
+        F, P = a @ a.T + np.eye(4), b @ b.T + np.eye(4)
+        ref = oracle.rel_change(F, P)
+        for c1, c2 in ((3.0, 1.0), (1.0, 0.2), (7.5, 1e-3)):
+            assert oracle.rel_change(c1 * F, c2 * P) == pytest.approx(ref, rel=1e-13)
+
+
+def test_fit_delta_compares_consecutive_iterates():
+    """The fit's recorded delta_t is the larger of the two factors' changes between the
+    iterates it returned after t-1 and t iterations (the first is +inf), and it goes
+    to zero at a fixed point: the factorial design reaches its closed form in one
+    iteration (see test_factorial_design_closed_form), so delta_2 = delta_3 = 0."""
+    X, G, _ = make_small_fit()
+    f = oracle.flipflop_fit(X, G, iters=6, keep_iterates=True)
+    assert math.isinf(f.deltas[0])
+    for t in range(1, 6):
+        (A1, B1), (A0, B0) = f.iterates[t], f.iterates[t - 1]
+        want = max(oracle.rel_change(A1, A0), oracle.rel_change(B1, B0))
+        assert f.deltas[t] == pytest.approx(want, rel=1e-12)
+    # the same iterates come back from fits of fewer iterations
+    f3 = oracle.flipflop_fit(X, G, iters=3)
+    assert np.allclose(f3.A, f.iterates[2][0], rtol=1e-12)
+    assert np.allclose(f3.B, f.iterates[2][1], rtol=1e-12)
+    Xf, Gf, _, _ = synth.factorial_design(8, 7, 4, 3, seed=22, dtype=torch.float64)
+    ff3 = oracle.flipflop_fit(Xf, Gf, iters=3)
+    assert max(ff3.deltas[1:]) < 1e-13
+
+
+def test_damped_fixed_point_satisfies_damped_stationary_equations():
+    """With damping lambda > 0 (Appendix B: each factor is damped when it is computed,
+    including between iterations) the iteration converges to a pair with
+        A propto damp(E[(g^T B^-1 g) x x^T], lambda),  B propto damp(E[(x^T A^-1 x) g g^T], lambda),
+    damp(F) = F + lambda mean(diag F) I, checked by brute force (explicit inverses and
+    outer products) at the returned pair, each equation up to a positive scale."""
+    N, n, m = 300, 5, 4
+    X = _correlated(N, n, seed=23, stream=0)
+    G = _correlated(N, m, seed=23, stream=1) * (1.0 + 0.7 * np.abs(X[:, 2:3]))
+    lam = 0.1
+    fit = oracle.flipflop_fit(X, G, iters=400, damping=lam)
+    assert fit.deltas[-1] < 1e-13
+    Ai, Bi = np.linalg.inv(fit.A), np.linalg.inv(fit.B)
+    q = np.array([x @ Ai @ x for x in X])
+    r = np.array([g @ Bi @ g for g in G])
+
+    def damped(F):
+        return F + lam * np.trace(F) / F.shape[0] * np.eye(F.shape[0])
+
+    A_rhs = damped(_brute_gram(X, r, 1.0))
+    B_rhs = damped(_brute_gram(G, q, 1.0))
+    for F, R in ((fit.A, A_rhs), (fit.B, B_rhs)):
+        Fh, Rh = F / np.trace(F), R / np.trace(R)
+        assert np.linalg.norm(Fh - Rh) / np.linalg.norm(Rh) < 1e-10
+    # the undamped stationary equations do not hold there
+    Ah = _brute_gram(X, r, 1.0)
+    assert np.linalg.norm(fit.A / np.trace(fit.A) - Ah / np.trace(Ah)) > 1e-4
+    # and the damped fixed point differs from the undamped one
+    f0 = oracle.flipflop_fit(X, G, iters=400)
+    assert oracle.kron_rel_err(fit.A, fit.B, f0.A, f0.B) > 1e-3
+
+
+def test_damping_is_homogeneous_so_it_commutes_with_the_rescale():
+    """damp(c F) = c damp(F) for c > 0: damping before or after the tr(A) = n rescale
+    gives the same pair, so the order of those two steps is not a reading that
+    matters; the one that does (damping inside the iteration, before the next
+    inversion) is pinned by the damped stationary equations above."""
+    F = np.array([[2.0, 0.5, 0.1], [0.5, 3.0, 0.2], [0.1, 0.2, 1.0]])
+    for c in (0.3, 2.0, 17.0):
+        assert np.allclose(oracle.damp(c * F, 0.1), c * oracle.damp(F, 0.1), rtol=1e-15)
+
+
+def test_row_blocks_do_not_change_the_fit():
+    """The expectations are accumulated over blocks of rows; any block size gives the
+    same fit (up to the order of the additions), including a ragged last block."""
+    X, G, _ = make_small_fit()
+    f_all = oracle.flipflop_fit(X, G, iters=5)
+    f_7 = oracle.flipflop_fit(X, G, iters=5, rows=7)
+    f_64 = oracle.flipflop_fit(X, G, iters=5, rows=64)
+    def rel(P, Q):
+        return np.linalg.norm(P - Q) / np.linalg.norm(Q)
+
+    for f in (f_7, f_64):
+        assert rel(f.A, f_all.A) < 1e-12 and rel(f.B, f_all.B) < 1e-12
+        assert np.allclose(f.loglik, f_all.loglik, rtol=1e-12)
+    # bf16 samples held as torch tensors are widened block by block
+    Xb = torch.from_numpy(X).to(torch.bfloat16)
+    Gb = torch.from_numpy(G).to(torch.bfloat16)
+    fb = oracle.flipflop_fit(Xb, Gb, iters=3, rows=33)
+    fr = oracle.flipflop_fit(oracle.as_f64(Xb), oracle.as_f64(Gb), iters=3)
+    assert rel(fb.A, fr.A) < 1e-12 and rel(fb.B, fr.B) < 1e-12
+
+
 def test_tol_stops_early():
     N, n, m = 300, 4, 3
     X = _correlated(N, n, seed=13, stream=0)
