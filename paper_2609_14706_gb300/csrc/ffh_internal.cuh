@@ -6,9 +6,40 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "../../include/ffh.h"
 
 namespace ffh {
+
+// ---------------------------------------------------------------------------
+// per-device one-time set-up
+// ---------------------------------------------------------------------------
+// A kernel's dynamic shared-memory limit is an attribute of the current device's
+// context, so it is raised once per device, not once per process.  Bit i of `bits`
+// records device i (safe to read and set from several host threads; devices >= 64
+// repeat the set-up on every call, which is correct, only slower).
+struct PerDeviceOnce {
+  std::atomic<unsigned long long> bits{0};
+  bool done(int dev) const {
+    return dev >= 0 && dev < 64 && ((bits.load(std::memory_order_acquire) >> dev) & 1ull);
+  }
+  void set(int dev) {
+    if (dev >= 0 && dev < 64) bits.fetch_or(1ull << dev, std::memory_order_acq_rel);
+  }
+};
+
+// cudaFuncAttributeMaxDynamicSharedMemorySize = bytes for `func` on the current device,
+// once per device (two threads may both set it the first time: same value, harmless).
+inline cudaError_t smem_attr_once(const void* func, int bytes, PerDeviceOnce& once) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (once.done(dev)) return cudaSuccess;
+  e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) once.set(dev);
+  return e;
+}
 
 // ---------------------------------------------------------------------------
 // device status block (one per handle, in the workspace)

@@ -54,15 +54,16 @@ static cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
 }
 
 static PFN_cuTensorMapEncodeTiled_v12000 encode_fn_chol() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (!fn) {
+  // the driver entry point is the same for every device; looked up once, thread-safely
+  static const PFN_cuTensorMapEncodeTiled_v12000 fn = []() {
     void* p = nullptr;
     cudaDriverEntryPointQueryResult q;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
                                          &q) == cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  }
+      return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    return (PFN_cuTensorMapEncodeTiled_v12000) nullptr;
+  }();
   return fn;
 }
 
@@ -436,12 +437,10 @@ static cudaError_t gemm_tc(const Split& A, const Split& B, int nseg, const int a
               map_epi_3d(&lm, out_split->p + out_split->kpad, true, (uint64_t)N, (uint64_t)M,
                          (uint64_t)batch, pitch, zs);
   }
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         gt::SMEM_BYTES);
+  static PerDeviceOnce attr;
+  {
+    cudaError_t e = smem_attr_once((const void*)k_gemm_tc, gt::SMEM_BYTES, attr);
     if (e != cudaSuccess) return e;
-    attr = true;
   }
   GemmTcArgs g{};
   g.C = C;
@@ -702,12 +701,10 @@ static cudaError_t syrk_tc(const Split& A, const int a_seg[3], const int b_seg[3
   if (!map_bf16_kmajor(&am, A.p, (uint64_t)2 * A.kpad, (uint64_t)A.rows_pad * A.batch,
                        (uint64_t)2 * A.kpad, sy::BM))
     return cudaErrorInvalidValue;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_syrk_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         sy::SMEM_BYTES);
+  static PerDeviceOnce attr;
+  {
+    cudaError_t e = smem_attr_once((const void*)k_syrk_tc, sy::SMEM_BYTES, attr);
     if (e != cudaSuccess) return e;
-    attr = true;
   }
   SyrkArgs g{};
   const int ntm = (M + sy::BM - 1) / sy::BM;
@@ -1286,13 +1283,8 @@ static cudaError_t cholesky_tc_body(const float* F, int64_t d, int64_t ldf, floa
     sb[i] = reinterpret_cast<__nv_bfloat16*>(wp);
     wp += up((size_t)rows_cap * 2 * kmax * 2);
   }
-  static bool attr = false;
-  if (!attr) {
-    if ((e = cudaFuncSetAttribute(k_chol_leaf, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  LB_SMEM)) != cudaSuccess)
-      return e;
-    attr = true;
-  }
+  static PerDeviceOnce attr;
+  if ((e = smem_attr_once((const void*)k_chol_leaf, LB_SMEM, attr)) != cudaSuccess) return e;
   if ((e = cudaMemcpy2DAsync(W, d * 4, F, ldf * 4, d * 4, d, cudaMemcpyDeviceToDevice, s)) !=
       cudaSuccess)
     return e;

@@ -27,15 +27,16 @@ using namespace ptx;
 static constexpr uint64_t kTfWaitNs = 4000000000ull;
 
 static PFN_cuTensorMapEncodeTiled_v12000 encode_fn_mx() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (!fn) {
+  // the driver entry point is the same for every device; looked up once, thread-safely
+  static const PFN_cuTensorMapEncodeTiled_v12000 fn = []() {
     void* p = nullptr;
     cudaDriverEntryPointQueryResult q;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
                                          &q) == cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  }
+      return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    return (PFN_cuTensorMapEncodeTiled_v12000) nullptr;
+  }();
   return fn;
 }
 
@@ -285,16 +286,11 @@ cudaError_t launch_transform_tc(const __nv_bfloat16* M, int64_t d, int64_t ldm,
     if (!map2d_bf16(&gm, Gb, (uint64_t)n, (uint64_t)(nk * m), (uint64_t)n, 64, tf::BK))
       return cudaErrorInvalidValue;
   }
-  static bool attr[2] = {false, false};
-  if (!attr[b_update ? 0 : 1]) {
-    cudaError_t e = b_update ? cudaFuncSetAttribute(k_transform_tc<false>,
-                                                    cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                    tf::SMEM_BYTES)
-                             : cudaFuncSetAttribute(k_transform_tc<true>,
-                                                    cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                    tf::SMEM_BYTES);
+  static PerDeviceOnce attr[2];
+  {
+    const void* fn = b_update ? (const void*)k_transform_tc<false> : (const void*)k_transform_tc<true>;
+    cudaError_t e = smem_attr_once(fn, tf::SMEM_BYTES, attr[b_update ? 0 : 1]);
     if (e != cudaSuccess) return e;
-    attr[b_update ? 0 : 1] = true;
   }
   TransformArgs a;
   a.V = V;

@@ -40,15 +40,16 @@ static constexpr uint64_t kFaultWaitBudgetNs = 20000000ull;   // 20 ms (fault in
 // tensor maps
 // ---------------------------------------------------------------------------
 static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (!fn) {
+  // the driver entry point is the same for every device; looked up once, thread-safely
+  static const PFN_cuTensorMapEncodeTiled_v12000 fn = []() {
     void* p = nullptr;
     cudaDriverEntryPointQueryResult q;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
                                          &q) == cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  }
+      return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    return (PFN_cuTensorMapEncodeTiled_v12000) nullptr;
+  }();
   return fn;
 }
 
@@ -415,12 +416,10 @@ cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t
   } else if (!make_map_bf16(&amap, Va, (uint64_t)d, (uint64_t)N, (uint64_t)lda, 64, gram::BK)) {
     return cudaErrorInvalidValue;
   }
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_gram_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         gram::SMEM_BYTES);
+  static PerDeviceOnce attr;
+  {
+    cudaError_t e = smem_attr_once((const void*)k_gram_tc, gram::SMEM_BYTES, attr);
     if (e != cudaSuccess) return e;
-    attr = true;
   }
   GramArgs a;
   a.w = w_padded;
@@ -699,12 +698,10 @@ cudaError_t launch_qform_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_
     return cudaErrorInvalidValue;
   if (!make_map_bf16(&mmap, M, (uint64_t)d, (uint64_t)d, (uint64_t)ldm, qf::BK, qf::BN))
     return cudaErrorInvalidValue;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_qform_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         qf::SMEM_BYTES);
+  static PerDeviceOnce attr;
+  {
+    cudaError_t e = smem_attr_once((const void*)k_qform_tc, qf::SMEM_BYTES, attr);
     if (e != cudaSuccess) return e;
-    attr = true;
   }
   QformArgs a;
   a.q = q;

@@ -1,0 +1,164 @@
+"""Portable seeded samples: the same bytes on any host and on any device.
+
+The default generators (``workloads.py``) draw with torch's device generators, whose
+streams differ between the CPU and a GPU.  The full-size parity runs need the fp64
+oracle (on one machine's host cores) and the CUDA fit (on a GPU machine) to see the
+same samples, so this module draws them in a way that does not depend on the machine:
+
+* every normal variate comes from numpy's PCG64 generator (integer state), seeded by a
+  SeedSequence of (seed, stream[, chunk]), in fp64, one generator per fixed chunk of
+  rows, so the bytes do not depend on how many threads draw them;
+* the mixing x = S z and every scaling are done in fp64, on the host or on a GPU;
+* the result is rounded once to fp32 and then, for bf16 workloads, to bf16 (both
+  round-to-nearest-even).
+
+fp64 arithmetic done in another order (another BLAS, a GPU's) moves a value by a few
+units in its last place; that changes the rounded value only when the value lies that
+close to a rounding midpoint, about once in 10^13 bf16 elements (10^8 for fp32
+elements).  ``sha256`` digests the bytes so that both sides can confirm they saw the
+same samples.
+
+The recipe is the one of ``workloads.py`` (power-law covariances with a Haar-like
+rotation, outlier channels, multivariate Student-t inputs, g scale); only the random
+streams differ.  This module holds none of the estimator's arithmetic.
+"""
+from __future__ import annotations
+
+import hashlib
+import os
+from concurrent.futures import ThreadPoolExecutor
+from typing import Optional
+
+import numpy as np
+import torch
+
+from .workloads import Workload, exponent_for_condition
+
+# rows per generator chunk; fixed, so the bytes never depend on memory or threads
+CHUNK_ROWS = 8192
+
+# stream keys (a namespace of their own: 1000 + k)
+_QX, _QG, _ZX, _ZG, _OUT, _W, _QA, _QB, _ZK = (1000 + k for k in range(9))
+
+
+def _rng(seed: int, *key: int) -> np.random.Generator:
+    return np.random.Generator(np.random.PCG64(np.random.SeedSequence([int(seed), *map(int, key)])))
+
+
+def orthogonal64(d: int, seed: int, stream: int) -> np.ndarray:
+    """Seeded orthogonal d x d matrix (fp64): QR of a Gaussian matrix, signs fixed so
+    that R has a positive diagonal (a Haar-distributed rotation)."""
+    a = _rng(seed, stream).standard_normal((d, d))
+    q, r = np.linalg.qr(a)
+    s = np.sign(np.diag(r))
+    s[s == 0] = 1.0
+    return q * s[None, :]
+
+
+def sqrt_cov64(d: int, exponent: float, seed: int, stream: int) -> np.ndarray:
+    """S = Q diag(lambda)^{1/2} (fp64), lambda_i = i^-exponent, so S S^T = Q diag(lambda) Q^T."""
+    lam = np.arange(1, d + 1, dtype=np.float64) ** (-float(exponent))
+    return orthogonal64(d, seed, stream) * np.sqrt(lam)[None, :]
+
+
+def _threads() -> int:
+    try:
+        n = len(os.sched_getaffinity(0))
+    except Exception:
+        n = os.cpu_count() or 1
+    return max(1, min(16, n))
+
+
+def _round_to(x64: torch.Tensor, dtype: torch.dtype) -> torch.Tensor:
+    x32 = x64.to(torch.float32)
+    return x32 if dtype == torch.float32 else x32.to(dtype)
+
+
+def rank_one_samples(wl: Workload, seed: int = 0, device="cpu", N: Optional[int] = None):
+    """(X, G) of the rank-one workload `wl` on `device`, dtype wl.dtype, drawn portably.
+
+    x_k = S_x z_k (Gaussian) or S_x z_k / sqrt(w_k / nu) (multivariate Student-t,
+    w_k a sum of nu squared normals), then the outlier channels are scaled;
+    g_k = g_scale S_g z'_k.  All of it in fp64, one rounding at the end."""
+    assert wl.kind == "rank_one"
+    N = wl.N if N is None else int(N)
+    dev = torch.device(device)
+    SxT = torch.from_numpy(sqrt_cov64(wl.n, wl.x_exponent, seed, _QX).T.copy()).to(dev)
+    SgT = torch.from_numpy(sqrt_cov64(wl.m, wl.g_exponent, seed, _QG).T.copy()).to(dev)
+    col = np.ones(wl.n)
+    if wl.x_outliers:
+        col[_rng(seed, _OUT).permutation(wl.n)[: wl.x_outliers]] = wl.outlier_scale
+    col_t = torch.from_numpy(col).to(dev)
+    X = torch.empty(N, wl.n, device=dev, dtype=wl.torch_dtype)
+    G = torch.empty(N, wl.m, device=dev, dtype=wl.torch_dtype)
+    nu = int(wl.student_nu)
+
+    def draw(c: int):
+        r0 = c * CHUNK_ROWS
+        rows = min(N, r0 + CHUNK_ROWS) - r0
+        zx = _rng(seed, _ZX, c).standard_normal((rows, wl.n))
+        zg = _rng(seed, _ZG, c).standard_normal((rows, wl.m))
+        f = None
+        if nu:
+            u = _rng(seed, _W, c).standard_normal((rows, nu))
+            w = u[:, 0] * u[:, 0]
+            for j in range(1, nu):          # fixed summation order
+                w = w + u[:, j] * u[:, j]
+            f = 1.0 / np.sqrt(w / nu)
+        return r0, rows, zx, zg, f
+
+    nchunks = (N + CHUNK_ROWS - 1) // CHUNK_ROWS
+    with ThreadPoolExecutor(_threads()) as ex:
+        ahead = max(2, _threads())
+        futs = [ex.submit(draw, c) for c in range(min(nchunks, ahead))]
+        for c in range(nchunks):
+            r0, rows, zx, zg, f = futs[c].result()
+            futs[c] = None
+            if c + ahead < nchunks:
+                futs.append(ex.submit(draw, c + ahead))
+            x = torch.from_numpy(zx).to(dev) @ SxT
+            if f is not None:
+                x = x * torch.from_numpy(f).to(dev).unsqueeze(1)
+            x = x * col_t
+            X[r0:r0 + rows] = _round_to(x, wl.torch_dtype)
+            g = (torch.from_numpy(zg).to(dev) @ SgT) * wl.g_scale
+            G[r0:r0 + rows] = _round_to(g, wl.torch_dtype)
+            del x, g
+    return X, G
+
+
+def matrix_normal_factors(wl: Workload, seed: int = 0):
+    """(S_A, S_B) in fp64 on the host for the matrix workload: S S^T = A0 (n x n), B0
+    (m x m), power-law spectra with condition number wl.cond."""
+    SA = sqrt_cov64(wl.n, exponent_for_condition(wl.n, wl.cond), seed, _QA)
+    SB = sqrt_cov64(wl.m, exponent_for_condition(wl.m, wl.cond), seed, _QB)
+    return SA, SB
+
+
+def matrix_sample_chunk(wl: Workload, seed: int, k0: int, k1: int, SA_t: torch.Tensor,
+                        SB_t: torch.Tensor) -> torch.Tensor:
+    """Samples k0..k1-1 of the matrix workload, G_k = S_B Z_k S_A^T (fp64 on the device
+    of SA_t, rounded once to wl.dtype).  Samples are drawn per generator chunk of
+    CHUNK_ROWS // 64 samples, so any k0..k1 reproduce the same bytes."""
+    per = max(1, CHUNK_ROWS // 64)
+    out = []
+    dev = SA_t.device
+    c0, c1 = k0 // per, (k1 - 1) // per
+    for c in range(c0, c1 + 1):
+        a = c * per
+        rows = min(wl.N, a + per) - a
+        z = _rng(seed, _ZK, c).standard_normal((rows, wl.m, wl.n))
+        lo, hi = max(k0, a) - a, min(k1, a + rows) - a
+        zt = torch.from_numpy(z[lo:hi]).to(dev)
+        out.append(_round_to(torch.matmul(torch.matmul(SB_t, zt), SA_t.t()), wl.torch_dtype))
+    return torch.cat(out, 0)
+
+
+def sha256(*tensors: torch.Tensor, chunk_bytes: int = 1 << 28) -> str:
+    """Digest of the raw bytes of the tensors, in order (row-major, as stored)."""
+    h = hashlib.sha256()
+    for t in tensors:
+        flat = t.contiguous().view(-1).view(torch.uint8)
+        for i in range(0, flat.numel(), chunk_bytes):
+            h.update(flat[i:i + chunk_bytes].cpu().numpy().tobytes())
+    return h.hexdigest()

@@ -118,12 +118,15 @@ def exponent_for_condition(d: int, cond: float) -> float:
 
 
 def orthogonal(d: int, gen: torch.Generator, device) -> torch.Tensor:
-    """Seeded orthogonal d x d matrix (fp32): QR of a Gaussian matrix, signs fixed."""
+    """Seeded orthogonal d x d matrix (fp32): QR of a Gaussian matrix, signs fixed.
+
+    The Gaussian matrix is drawn on the generator's device; the QR runs on the host in
+    fp64 (no device linear-algebra library is needed to draw inputs)."""
     a = torch.randn(d, d, generator=gen, device=device, dtype=torch.float32)
-    q, r = torch.linalg.qr(a)
+    q, r = torch.linalg.qr(a.to("cpu", torch.float64))
     s = torch.sign(torch.diagonal(r))
     s[s == 0] = 1
-    return q * s.unsqueeze(0)
+    return (q * s.unsqueeze(0)).to(device=device, dtype=torch.float32)
 
 
 def sqrt_cov(d: int, exponent: float, gen: torch.Generator, device) -> torch.Tensor:

