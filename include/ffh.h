@@ -87,8 +87,7 @@ typedef struct {
                               NULL: A_0 = I_n (Appendix B) */
   int32_t final_loglik;    /* 1: also evaluate the log-likelihood at the returned (A, B)
                               (one more Cholesky and quadratic-form pass) */
-  int32_t kernel;          /* 0: tensor-core kernels (tcgen05); 1: CUDA-core kernels
-                              (slower; for cross-checking the tensor-core path) */
+  int32_t reserved0;       /* must be zero */
   int32_t fault;           /* FFH_FAULT_* (tests only) */
   int32_t profile;         /* 1: time the Gram, quadratic-form and Cholesky kernels with
                               CUDA events on the handle's stream (see ffh_get_timings) */

@@ -35,7 +35,7 @@ FAULT_NONE, FAULT_OOM, FAULT_BAD_PIVOT, FAULT_LOST_COPY = 0, 1, 2, 3
 class ffh_options(ctypes.Structure):
     _fields_ = [("dtype", ctypes.c_int32), ("damping", ctypes.c_float),
                 ("variant", ctypes.c_int32), ("init_A", ctypes.c_void_p),
-                ("final_loglik", ctypes.c_int32), ("kernel", ctypes.c_int32),
+                ("final_loglik", ctypes.c_int32), ("reserved0", ctypes.c_int32),
                 ("fault", ctypes.c_int32), ("profile", ctypes.c_int32),
                 ("reserved", ctypes.c_int32 * 4)]
 
@@ -129,7 +129,7 @@ class Handle:
 
     def __init__(self, dtype="bf16", damping: float = 0.0, variant: str = "flipflop",
                  init_A: Optional[torch.Tensor] = None, final_loglik: bool = False,
-                 kernel: str = "tc", fault: int = 0, profile: bool = False,
+                 fault: int = 0, profile: bool = False,
                  stream: Optional[torch.cuda.Stream] = None):
         self._lib = load_library()
         self._keep = []
@@ -142,7 +142,6 @@ class Handle:
             self._keep.append(init_A)
             self.opts.init_A = init_A.data_ptr()
         self.opts.final_loglik = int(bool(final_loglik))
-        self.opts.kernel = {"tc": 0, "simt": 1}[kernel]
         self.opts.fault = int(fault)
         self.opts.profile = int(bool(profile))
         self.stream = stream if stream is not None else torch.cuda.current_stream()

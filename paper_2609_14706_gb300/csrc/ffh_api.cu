@@ -177,8 +177,8 @@ ffh_status read_status(ffh_t h, DevStatus* st_dev) {
   return FFH_OK;
 }
 
-// Input staging: a device bf16 view of V (for the tensor-core kernels) and a device
-// view in the caller's dtype (for the CUDA-core kernels).
+// Input staging: a device bf16 view of V (the tensor-core operand) and a device view in
+// the caller's dtype (read by the A_0 = I row sums).
 struct Staged {
   const __nv_bfloat16* bf = nullptr;
   int64_t ld_bf = 0;
@@ -256,7 +256,7 @@ ffh_status validate_opt(ffh_t h) {
     return fail(h, FFH_ERR_INVALID_ARG, "damping must be finite and >= 0");
   if (o.variant < FFH_FLIPFLOP || o.variant > FFH_MARGINAL)
     return fail(h, FFH_ERR_INVALID_ARG, "bad variant %d", o.variant);
-  if (o.kernel != 0 && o.kernel != 1) return fail(h, FFH_ERR_INVALID_ARG, "bad kernel %d", o.kernel);
+  if (o.reserved0 != 0) return fail(h, FFH_ERR_INVALID_ARG, "reserved option field must be zero");
   return FFH_OK;
 }
 
@@ -299,73 +299,52 @@ ffh_status gram(ffh_t h, const Staged& V, int64_t N, int64_t d, const float* w_p
                 float* C, float* partial, const GramTables& gt, DevStatus* st,
                 __nv_bfloat16* vw = nullptr) {
   cudaEvent_t t0 = prof_begin(h);
-  if (h->opt.kernel == 1) {
-    CK(launch_gram_simt(V.raw, h->opt.dtype, N, d, V.ld_raw, w_padded, scale, C, d, h->stream));
-    prof_end(h, PROF_GRAM, t0);
-  } else {
-    cudaEvent_t t1 = t0 ? next_event(h) : nullptr;
-    const __nv_bfloat16* va = nullptr;
-    if (vw && w_padded) {
-      CK(launch_scale_rows(V.bf, V.ld_bf, N, d, w_padded, vw, V.ld_bf, h->stream));
-      va = vw;
-      w_padded = nullptr;
-    }
-    CK(launch_gram_tc(V.bf, N, d, V.ld_bf, w_padded, scale, C, d, partial, gt.tiles, gt.lut,
-                      gt.plan, st, h->opt.fault, h->stream, t1, va, V.ld_bf));
-    prof_end(h, PROF_GRAM, t0, t1);
+  cudaEvent_t t1 = t0 ? next_event(h) : nullptr;
+  const __nv_bfloat16* va = nullptr;
+  if (vw && w_padded) {
+    CK(launch_scale_rows(V.bf, V.ld_bf, N, d, w_padded, vw, V.ld_bf, h->stream));
+    va = vw;
+    w_padded = nullptr;
   }
+  CK(launch_gram_tc(V.bf, N, d, V.ld_bf, w_padded, scale, C, d, partial, gt.tiles, gt.lut,
+                    gt.plan, st, h->opt.fault, h->stream, t1, va, V.ld_bf));
+  prof_end(h, PROF_GRAM, t0, t1);
   return FFH_OK;
 }
 
 // q_k = ||L^T v_k||^2 = v_k^T F v_k for F = L L^T (the Frobenius variant's weights)
 ffh_status qform_fwd(ffh_t h, const Staged& V, int64_t N, int64_t d, const float* L,
-                     const float* F, __nv_bfloat16* Mb, float* q, DevStatus* st) {
-  if (h->opt.kernel == 1) {
-    cudaEvent_t t0 = prof_begin(h);
-    CK(launch_fwd_qform_simt(V.raw, h->opt.dtype, N, d, V.ld_raw, F, d, q, h->stream));
-    prof_end(h, PROF_QFORM, t0);
-  } else {
-    const int64_t ldm = pad8(d);
-    CK(launch_lowerT_to_bf16(L, d, d, Mb, ldm, h->stream));
-    cudaEvent_t t0 = prof_begin(h);
-    CK(launch_qform_tc(V.bf, N, d, V.ld_bf, Mb, ldm, q, st, h->stream, true));
-    prof_end(h, PROF_QFORM, t0);
-  }
+                     __nv_bfloat16* Mb, float* q, DevStatus* st) {
+  const int64_t ldm = pad8(d);
+  CK(launch_lowerT_to_bf16(L, d, d, Mb, ldm, h->stream));
+  cudaEvent_t t0 = prof_begin(h);
+  CK(launch_qform_tc(V.bf, N, d, V.ld_bf, Mb, ldm, q, st, h->stream, true));
+  prof_end(h, PROF_QFORM, t0);
   return FFH_OK;
 }
 
 ffh_status qform(ffh_t h, const Staged& V, int64_t N, int64_t d, const float* Linv,
                  __nv_bfloat16* Mb, float* q, DevStatus* st) {
-  if (h->opt.kernel == 1) {
-    cudaEvent_t t0 = prof_begin(h);
-    CK(launch_qform_simt(V.raw, h->opt.dtype, N, d, V.ld_raw, Linv, d, q, h->stream));
-    prof_end(h, PROF_QFORM, t0);
-  } else {
-    const int64_t ldm = pad8(d);
-    CK(launch_lower_to_bf16(Linv, d, d, Mb, ldm, h->stream));
-    cudaEvent_t t0 = prof_begin(h);
-    CK(launch_qform_tc(V.bf, N, d, V.ld_bf, Mb, ldm, q, st, h->stream));
-    prof_end(h, PROF_QFORM, t0);
-  }
+  const int64_t ldm = pad8(d);
+  CK(launch_lower_to_bf16(Linv, d, d, Mb, ldm, h->stream));
+  cudaEvent_t t0 = prof_begin(h);
+  CK(launch_qform_tc(V.bf, N, d, V.ld_bf, Mb, ldm, q, st, h->stream));
+  prof_end(h, PROF_QFORM, t0);
   return FFH_OK;
 }
 
 // Cholesky factor and inverse of F (d x d), timed as one region.
-ffh_status chol(ffh_t h, const float* F, int64_t d, float* L, float* Linv, float* work, float* DI,
+ffh_status chol(ffh_t h, const float* F, int64_t d, float* L, float* Linv, float* work,
                 DevStatus* st, int fault) {
   cudaEvent_t t0 = prof_begin(h);
-  if (h->opt.kernel == 1) {
-    CK(launch_cholesky(F, d, d, L, Linv, work, DI, st, fault, h->stream));
-  } else {
-    if (!h->chol_cs.crit) {
-      const cudaError_t e = chol_streams_init(&h->chol_cs);
-      if (e != cudaSuccess) {
-        chol_streams_destroy(&h->chol_cs);
-        return fail(h, FFH_ERR_CUDA, "Cholesky streams: %s", cudaGetErrorString(e));
-      }
+  if (!h->chol_cs.crit) {
+    const cudaError_t e = chol_streams_init(&h->chol_cs);
+    if (e != cudaSuccess) {
+      chol_streams_destroy(&h->chol_cs);
+      return fail(h, FFH_ERR_CUDA, "Cholesky streams: %s", cudaGetErrorString(e));
     }
-    CK(launch_cholesky_tc(F, d, d, L, Linv, work, st, fault, h->stream, &h->chol_cs));
   }
+  CK(launch_cholesky_tc(F, d, d, L, Linv, work, st, fault, h->stream, &h->chol_cs));
   prof_end(h, PROF_CHOL, t0);
   return FFH_OK;
 }
@@ -405,24 +384,22 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
   if (N < std::max(n, m) && h->opt.damping == 0.f)
     return fail(h, FFH_ERR_RANK, "N = %lld < max(n, m) = %lld without damping",
                 (long long)N, (long long)std::max(n, m));
-  const bool tc = h->opt.kernel == 0;
   const int dtype = h->opt.dtype;
   const bool x_dev = is_device_ptr(X), g_dev = is_device_ptr(G);
   const bool init = h->opt.init_A != nullptr;
   const int64_t D = std::max(n, m);
   const int64_t Npad = (N + 63) / 64 * 64 + 64;
-  const int nt = (int)((D + 63) / 64);
 
   GramPlan pn = gram_plan(N, n, num_sms()), pm = gram_plan(N, m, num_sms());
   auto layout = [&](Carve& c, DevStatus** st, IterRecord** recs, __nv_bfloat16** Xb,
                     __nv_bfloat16** Gb, float** stage, float** q, float** r, float** A2,
                     float** B2, float** L, float** Linv, __nv_bfloat16** Mb, float** work,
-                    float** DI, int2** tn, int** ln, int2** tm, int** lm, float** partial,
+                    int2** tn, int** ln, int2** tm, int** lm, float** partial,
                     double** trb, __nv_bfloat16** Vw) {
     *st = c.take<DevStatus>(1);
     *recs = c.take<IterRecord>(iters + 2);
-    const bool xcopy = (dtype == FFH_F32 && tc) || (dtype == FFH_BF16 && !x_dev);
-    const bool gcopy = (dtype == FFH_F32 && tc) || (dtype == FFH_BF16 && !g_dev);
+    const bool xcopy = dtype == FFH_F32 || (dtype == FFH_BF16 && !x_dev);
+    const bool gcopy = dtype == FFH_F32 || (dtype == FFH_BF16 && !g_dev);
     *Xb = xcopy ? c.take<__nv_bfloat16>((size_t)N * pad8(n)) : nullptr;
     *Gb = gcopy ? c.take<__nv_bfloat16>((size_t)N * pad8(m)) : nullptr;
     const bool host_f32 = dtype == FFH_F32 && (!x_dev || !g_dev);
@@ -434,33 +411,31 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
     *L = c.take<float>((size_t)D * D);
     *Linv = c.take<float>((size_t)D * D);
     *Mb = c.take<__nv_bfloat16>((size_t)D * pad8(D));
-    *work = c.take<float>(std::max(cholesky_work_floats(D), cholesky_tc_work_bytes(D) / 4 + 1));
-    *DI = c.take<float>((size_t)nt * 64 * 64);
+    *work = c.take<float>(cholesky_tc_work_bytes(D) / 4 + 1);
     *tn = c.take<int2>(gram_tile_table_bytes(n) / sizeof(int2) + 1);
     *ln = c.take<int>(gram_tile_table_bytes(n) / sizeof(int) + 1);
     *tm = c.take<int2>(gram_tile_table_bytes(m) / sizeof(int2) + 1);
     *lm = c.take<int>(gram_tile_table_bytes(m) / sizeof(int) + 1);
-    *partial = tc ? c.take<float>(std::max(gram_partial_bytes(pn), gram_partial_bytes(pm)) / 4)
-                  : nullptr;
+    *partial = c.take<float>(std::max(gram_partial_bytes(pn), gram_partial_bytes(pm)) / 4);
     *trb = c.take<double>(8);
-    *Vw = tc ? c.take<__nv_bfloat16>((size_t)N * pad8(D)) : nullptr;
+    *Vw = c.take<__nv_bfloat16>((size_t)N * pad8(D));
   };
   DevStatus* st;
   IterRecord* recs;
   __nv_bfloat16 *Xb, *Gb, *Mb, *Vw;
-  float *stage, *q, *r, *A2, *B2, *L, *Linv, *work, *DI, *partial;
+  float *stage, *q, *r, *A2, *B2, *L, *Linv, *work, *partial;
   int2 *tn, *tm;
   int *ln, *lm;
   double* trb;
   {
     Carve c(nullptr);
-    layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &DI, &tn,
+    layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &tn,
            &ln, &tm, &lm, &partial, &trb, &Vw);
     ffh_status es = ensure_ws(h, c.off + 1024);
     if (es) return es;
   }
   Carve c(h->ws);
-  layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &DI, &tn, &ln,
+  layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &tn, &ln,
          &tm, &lm, &partial, &trb, &Vw);
   cudaStream_t s = h->stream;
   CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
@@ -468,7 +443,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
   CK(cudaMemsetAsync(q, 0, sizeof(float) * Npad, s));
   CK(cudaMemsetAsync(r, 0, sizeof(float) * Npad, s));
   GramTables gtn, gtm;
-  if (tc) {
+  {
     ffh_status es = setup_tables(h, N, n, &gtn, tn, ln);
     if (es) return es;
     es = setup_tables(h, N, m, &gtm, tm, lm);
@@ -521,12 +496,12 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
     if (t == 1 && !init) {
       CK(launch_rowsumsq(xs.raw, dtype, N, n, xs.ld_raw, q, s));
     } else if (frob) {
-      es = chol(h, A[cur], n, L, nullptr, work, DI, st, 0);
+      es = chol(h, A[cur], n, L, nullptr, work, st, 0);
       if (es) return es;
-      es = qform_fwd(h, xs, N, n, L, A[cur], Mb, q, st);
+      es = qform_fwd(h, xs, N, n, L, Mb, q, st);
       if (es) return es;
     } else {
-      es = chol(h, A[cur], n, L, Linv, work, DI, st, 0);
+      es = chol(h, A[cur], n, L, Linv, work, st, 0);
       if (es) return es;
       CK(cudaMemcpyAsync(&R->logdet_A_prev, &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
       if (t > 1)
@@ -544,12 +519,12 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
       CK(launch_scale_by_inv(B[nxt], m, trb + 4, s));
     }
     CK(launch_damp(B[nxt], m, m, lam, st, s));
-    es = chol(h, B[nxt], m, L, frob ? nullptr : Linv, work, DI, st,
+    es = chol(h, B[nxt], m, L, frob ? nullptr : Linv, work, st,
               (t == 1 && h->opt.fault == FFH_FAULT_BAD_PIVOT) ? FFH_FAULT_BAD_PIVOT : 0);
     if (es) return es;
     CK(cudaMemcpyAsync(&R->logdet_B, &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
     if (frob) {
-      es = qform_fwd(h, gs, N, m, L, B[nxt], Mb, r, st);
+      es = qform_fwd(h, gs, N, m, L, Mb, r, st);
     } else {
       es = qform(h, gs, N, m, Linv, Mb, r, st);
     }
@@ -586,7 +561,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
     }
   }
   if (h->opt.final_loglik && variant == FFH_FLIPFLOP) {
-    es = chol(h, A[cur], n, L, Linv, work, DI, st, 0);
+    es = chol(h, A[cur], n, L, Linv, work, st, 0);
     if (es) return es;
     CK(cudaMemcpyAsync(&recs[t_done].logdet_A, &st->logdet, sizeof(double),
                        cudaMemcpyDeviceToDevice, s));
@@ -620,7 +595,6 @@ extern "C" ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_
     return fail(h, FFH_ERR_INVALID_ARG, "need N, n, m, iters >= 1");
   if (n % 8 || m % 8) return fail(h, FFH_ERR_INVALID_ARG, "matrix samples need n, m multiples of 8");
   if (!(tol >= 0.f) || !std::isfinite(tol)) return fail(h, FFH_ERR_INVALID_ARG, "tol must be finite and >= 0");
-  if (h->opt.kernel != 0) return fail(h, FFH_ERR_UNSUPPORTED, "matrix samples need the tensor-core kernels");
   if (h->opt.variant != FFH_FLIPFLOP) return fail(h, FFH_ERR_UNSUPPORTED, "matrix samples: FlipFlop variant only");
   if (N * std::min(n, m) < std::max(n, m) && h->opt.damping == 0.f)
     return fail(h, FFH_ERR_RANK, "N min(n, m) < max(n, m) without damping");
@@ -634,10 +608,9 @@ extern "C" ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_
   const int64_t Kc = std::max<int64_t>(1, std::min<int64_t>(N, ((int64_t)1 << 29) / mn));
   const int64_t Kh = g_dev ? 0 : Kc;  // host staging (fp32) chunk
   GramPlan pa = gram_plan(Kc * m, n, num_sms()), pb = gram_plan(Kc * n, m, num_sms());
-  const int nt = (int)((D + 63) / 64);
   auto layout = [&](Carve& c, DevStatus** st, IterRecord** recs, __nv_bfloat16** Gb,
                     float** stage, __nv_bfloat16** V, float** A2, float** B2, float** Cc,
-                    float** L, float** Linv, __nv_bfloat16** Mb, float** work, float** DI,
+                    float** L, float** Linv, __nv_bfloat16** Mb, float** work,
                     int2** tn, int** ln, int2** tm, int** lm, float** partial, double** trb,
                     double** fro) {
     *st = c.take<DevStatus>(1);
@@ -651,8 +624,7 @@ extern "C" ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_
     *L = c.take<float>((size_t)D * D);
     *Linv = c.take<float>((size_t)D * D);
     *Mb = c.take<__nv_bfloat16>((size_t)D * D);
-    *work = c.take<float>(std::max(cholesky_work_floats(D), cholesky_tc_work_bytes(D) / 4 + 1));
-    *DI = c.take<float>((size_t)nt * 64 * 64);
+    *work = c.take<float>(cholesky_tc_work_bytes(D) / 4 + 1);
     *tn = c.take<int2>(gram_tile_table_bytes(n) / sizeof(int2) + 1);
     *ln = c.take<int>(gram_tile_table_bytes(n) / sizeof(int) + 1);
     *tm = c.take<int2>(gram_tile_table_bytes(m) / sizeof(int2) + 1);
@@ -664,19 +636,19 @@ extern "C" ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_
   DevStatus* st;
   IterRecord* recs;
   __nv_bfloat16 *Gb, *V, *Mb;
-  float *stage, *A2, *B2, *Cc, *L, *Linv, *work, *DI, *partial;
+  float *stage, *A2, *B2, *Cc, *L, *Linv, *work, *partial;
   int2 *tn, *tm;
   int *ln, *lm;
   double *trb, *fro;
   {
     Carve c(nullptr);
-    layout(c, &st, &recs, &Gb, &stage, &V, &A2, &B2, &Cc, &L, &Linv, &Mb, &work, &DI, &tn, &ln,
+    layout(c, &st, &recs, &Gb, &stage, &V, &A2, &B2, &Cc, &L, &Linv, &Mb, &work, &tn, &ln,
            &tm, &lm, &partial, &trb, &fro);
     ffh_status es = ensure_ws(h, c.off + 1024);
     if (es) return es;
   }
   Carve c(h->ws);
-  layout(c, &st, &recs, &Gb, &stage, &V, &A2, &B2, &Cc, &L, &Linv, &Mb, &work, &DI, &tn, &ln, &tm,
+  layout(c, &st, &recs, &Gb, &stage, &V, &A2, &B2, &Cc, &L, &Linv, &Mb, &work, &tn, &ln, &tm,
          &lm, &partial, &trb, &fro);
   cudaStream_t s = h->stream;
   CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
@@ -745,7 +717,7 @@ extern "C" ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_
     IterRecord* R = recs + t;
     const int nxt = cur ^ 1;
     // ---- M_A = chol(A_{t-1})^-1 (bf16)
-    es = chol(h, A[cur], n, L, Linv, work, DI, st, 0);
+    es = chol(h, A[cur], n, L, Linv, work, st, 0);
     if (es) return es;
     CK(cudaMemcpyAsync(&R->logdet_A_prev, &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
     if (t > 1) {
@@ -758,7 +730,7 @@ extern "C" ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_
     es = half(Mb, n, true, sB, B[nxt], gtm);
     if (es) return es;
     CK(launch_damp(B[nxt], m, m, lam, st, s, &R->shift_B));
-    es = chol(h, B[nxt], m, L, Linv, work, DI, st,
+    es = chol(h, B[nxt], m, L, Linv, work, st,
               (t == 1 && h->opt.fault == FFH_FAULT_BAD_PIVOT) ? FFH_FAULT_BAD_PIVOT : 0);
     if (es) return es;
     CK(cudaMemcpyAsync(&R->logdet_B, &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
@@ -790,7 +762,7 @@ extern "C" ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_
     }
   }
   if (h->opt.final_loglik) {
-    es = chol(h, A[cur], n, L, Linv, work, DI, st, 0);
+    es = chol(h, A[cur], n, L, Linv, work, st, 0);
     if (es) return es;
     CK(cudaMemcpyAsync(&recs[t_done].logdet_A, &st->logdet, sizeof(double),
                        cudaMemcpyDeviceToDevice, s));
@@ -879,15 +851,14 @@ extern "C" ffh_status ffh_weighted_gram(ffh_t h, const void* V, const float* w, 
     return fail(h, FFH_ERR_INVALID_ARG, "single-step calls take device pointers");
   const int dtype = h->opt.dtype;
   if (dtype == FFH_BF16 && d % 8) return fail(h, FFH_ERR_INVALID_ARG, "bf16 rows: d multiple of 8");
-  const bool tc = h->opt.kernel == 0;
   const int64_t Npad = (N + 63) / 64 * 64 + 64;
   GramPlan plan = gram_plan(N, d, num_sms());
   auto layout = [&](Carve& c, DevStatus** st, float** wp, __nv_bfloat16** Vb, float** partial,
                     int2** tiles, int** lut) {
     *st = c.take<DevStatus>(1);
     *wp = c.take<float>(Npad);
-    *Vb = (tc && dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(d)) : nullptr;
-    *partial = tc ? c.take<float>(gram_partial_bytes(plan) / 4) : nullptr;
+    *Vb = (dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(d)) : nullptr;
+    *partial = c.take<float>(gram_partial_bytes(plan) / 4);
     *tiles = c.take<int2>(gram_tile_table_bytes(d) / sizeof(int2) + 1);
     *lut = c.take<int>(gram_tile_table_bytes(d) / sizeof(int) + 1);
   };
@@ -916,10 +887,8 @@ extern "C" ffh_status ffh_weighted_gram(ffh_t h, const void* V, const float* w, 
   ffh_status es = stage_input(h, V, true, N, d, Vb, nullptr, &vs_);
   if (es) return es;
   GramTables gt;
-  if (tc) {
-    es = setup_tables(h, N, d, &gt, tiles, lut);
-    if (es) return es;
-  }
+  es = setup_tables(h, N, d, &gt, tiles, lut);
+  if (es) return es;
   es = gram(h, vs_, N, d, wuse, scale, C_out, partial, gt, st);
   if (es) return es;
   return read_status(h, st);
@@ -937,10 +906,9 @@ extern "C" ffh_status ffh_quad_form(ffh_t h, const void* V, const float* Linv, i
     return fail(h, FFH_ERR_INVALID_ARG, "single-step calls take device pointers");
   const int dtype = h->opt.dtype;
   if (dtype == FFH_BF16 && d % 8) return fail(h, FFH_ERR_INVALID_ARG, "bf16 rows: d multiple of 8");
-  const bool tc = h->opt.kernel == 0;
   auto layout = [&](Carve& c, DevStatus** st, __nv_bfloat16** Vb, __nv_bfloat16** Mb) {
     *st = c.take<DevStatus>(1);
-    *Vb = (tc && dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(d)) : nullptr;
+    *Vb = (dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(d)) : nullptr;
     *Mb = c.take<__nv_bfloat16>((size_t)d * pad8(d));
   };
   DevStatus* st;
@@ -970,28 +938,26 @@ extern "C" ffh_status ffh_cholesky(ffh_t h, const float* F, int64_t d, float* L_
   if (!is_device_ptr(F) || (L_out && !is_device_ptr(L_out)) ||
       (Linv_out && !is_device_ptr(Linv_out)))
     return fail(h, FFH_ERR_INVALID_ARG, "single-step calls take device pointers");
-  const int nt = (int)((d + 63) / 64);
-  auto layout = [&](Carve& c, DevStatus** st, float** L, float** Li, float** work, float** DI) {
+  auto layout = [&](Carve& c, DevStatus** st, float** L, float** Li, float** work) {
     *st = c.take<DevStatus>(1);
     *L = L_out ? nullptr : c.take<float>((size_t)d * d);
     *Li = c.take<float>((size_t)d * d);
-    *work = c.take<float>(std::max(cholesky_work_floats(d), cholesky_tc_work_bytes(d) / 4 + 1));
-    *DI = c.take<float>((size_t)nt * 64 * 64);
+    *work = c.take<float>(cholesky_tc_work_bytes(d) / 4 + 1);
   };
   DevStatus* st;
-  float *L, *Li, *work, *DI;
+  float *L, *Li, *work;
   {
     Carve c(nullptr);
-    layout(c, &st, &L, &Li, &work, &DI);
+    layout(c, &st, &L, &Li, &work);
     ffh_status es = ensure_ws(h, c.off + 1024);
     if (es) return es;
   }
   Carve c(h->ws);
-  layout(c, &st, &L, &Li, &work, &DI);
+  layout(c, &st, &L, &Li, &work);
   if (L_out) L = L_out;
   cudaStream_t s = h->stream;
   CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
-  ffh_status cs = chol(h, F, d, L, Linv_out ? Linv_out : (float*)nullptr, work, DI, st,
+  ffh_status cs = chol(h, F, d, L, Linv_out ? Linv_out : (float*)nullptr, work, st,
                        h->opt.fault == FFH_FAULT_BAD_PIVOT ? FFH_FAULT_BAD_PIVOT : 0);
   if (cs) return cs;
   (void)Li;
@@ -1009,31 +975,28 @@ extern "C" ffh_status ffh_rev_cholesky(ffh_t h, const float* F, int64_t d, float
   if (!F || d < 1) return fail(h, FFH_ERR_INVALID_ARG, "bad arguments");
   if (!is_device_ptr(F) || (L_out && !is_device_ptr(L_out)) || (Lt_out && !is_device_ptr(Lt_out)))
     return fail(h, FFH_ERR_INVALID_ARG, "WaterKron calls take device pointers");
-  const int nt = (int)((d + 63) / 64);
-  auto layout = [&](Carve& c, DevStatus** st, float** Fr, float** C, float** Ci, float** work,
-                    float** DI) {
+  auto layout = [&](Carve& c, DevStatus** st, float** Fr, float** C, float** Ci, float** work) {
     *st = c.take<DevStatus>(1);
     *Fr = c.take<float>((size_t)d * d);
     *C = c.take<float>((size_t)d * d);
     *Ci = c.take<float>((size_t)d * d);
-    *work = c.take<float>(std::max(cholesky_work_floats(d), cholesky_tc_work_bytes(d) / 4 + 1));
-    *DI = c.take<float>((size_t)nt * 64 * 64);
+    *work = c.take<float>(cholesky_tc_work_bytes(d) / 4 + 1);
   };
   DevStatus* st;
-  float *Fr, *C, *Ci, *work, *DI;
+  float *Fr, *C, *Ci, *work;
   {
     Carve c(nullptr);
-    layout(c, &st, &Fr, &C, &Ci, &work, &DI);
+    layout(c, &st, &Fr, &C, &Ci, &work);
     ffh_status es = ensure_ws(h, c.off + 1024);
     if (es) return es;
   }
   Carve c(h->ws);
-  layout(c, &st, &Fr, &C, &Ci, &work, &DI);
+  layout(c, &st, &Fr, &C, &Ci, &work);
   cudaStream_t s = h->stream;
   CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
   // C C^T = J F J;  L = J C^T J,  L^-1 = J C^-T J (column-normalised for Algorithms 1-2)
   CK(launch_reverse_sym(F, d, d, Fr, s));
-  ffh_status es = chol(h, Fr, d, C, Ci, work, DI, st,
+  ffh_status es = chol(h, Fr, d, C, Ci, work, st,
                        h->opt.fault == FFH_FAULT_BAD_PIVOT ? FFH_FAULT_BAD_PIVOT : 0);
   if (es) return es;
   if (L_out) CK(launch_rev_transpose(C, d, L_out, false, s));
@@ -1127,37 +1090,34 @@ extern "C" ffh_status ffh_phi_tilde(ffh_t h, const void* X, const void* G, int64
   const int dtype = h->opt.dtype;
   if (dtype == FFH_BF16 && (n % 8 || m % 8))
     return fail(h, FFH_ERR_INVALID_ARG, "bf16 rows must be 16-byte aligned: n, m multiples of 8");
-  const bool tc = h->opt.kernel == 0;
   const int64_t D = std::max(n, m);
   const int64_t Npad = (N + 63) / 64 * 64 + 64;
-  const int nt = (int)((D + 63) / 64);
   auto layout = [&](Carve& c, DevStatus** st, __nv_bfloat16** Xb, __nv_bfloat16** Gb, float** q,
                     float** r, float** L, float** Linv, __nv_bfloat16** Mb, float** work,
-                    float** DI, double** acc) {
+                    double** acc) {
     *st = c.take<DevStatus>(1);
-    *Xb = (tc && dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(n)) : nullptr;
-    *Gb = (tc && dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(m)) : nullptr;
+    *Xb = (dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(n)) : nullptr;
+    *Gb = (dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(m)) : nullptr;
     *q = c.take<float>(Npad);
     *r = c.take<float>(Npad);
     *L = c.take<float>((size_t)D * D);
     *Linv = c.take<float>((size_t)D * D);
     *Mb = c.take<__nv_bfloat16>((size_t)D * pad8(D));
-    *work = c.take<float>(std::max(cholesky_work_floats(D), cholesky_tc_work_bytes(D) / 4 + 1));
-    *DI = c.take<float>((size_t)nt * 64 * 64);
+    *work = c.take<float>(cholesky_tc_work_bytes(D) / 4 + 1);
     *acc = c.take<double>(4);
   };
   DevStatus* st;
   __nv_bfloat16 *Xb, *Gb, *Mb;
-  float *q, *r, *L, *Linv, *work, *DI;
+  float *q, *r, *L, *Linv, *work;
   double* acc;
   {
     Carve c(nullptr);
-    layout(c, &st, &Xb, &Gb, &q, &r, &L, &Linv, &Mb, &work, &DI, &acc);
+    layout(c, &st, &Xb, &Gb, &q, &r, &L, &Linv, &Mb, &work, &acc);
     ffh_status es = ensure_ws(h, c.off + 1024);
     if (es) return es;
   }
   Carve c(h->ws);
-  layout(c, &st, &Xb, &Gb, &q, &r, &L, &Linv, &Mb, &work, &DI, &acc);
+  layout(c, &st, &Xb, &Gb, &q, &r, &L, &Linv, &Mb, &work, &acc);
   cudaStream_t s = h->stream;
   CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
   Staged xs, gs;
@@ -1166,12 +1126,12 @@ extern "C" ffh_status ffh_phi_tilde(ffh_t h, const void* X, const void* G, int64
   es = stage_input(h, G, true, N, m, Gb, nullptr, &gs);
   if (es) return es;
   double ld[2] = {0, 0};
-  es = chol(h, A, n, L, Linv, work, DI, st, 0);
+  es = chol(h, A, n, L, Linv, work, st, 0);
   if (es) return es;
   CK(cudaMemcpyAsync(&acc[1], &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
   es = qform(h, xs, N, n, Linv, Mb, q, st);
   if (es) return es;
-  es = chol(h, B, m, L, Linv, work, DI, st, 0);
+  es = chol(h, B, m, L, Linv, work, st, 0);
   if (es) return es;
   CK(cudaMemcpyAsync(&acc[2], &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
   es = qform(h, gs, N, m, Linv, Mb, r, st);

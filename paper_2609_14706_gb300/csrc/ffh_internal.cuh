@@ -159,22 +159,11 @@ cudaError_t launch_lowerT_to_bf16(const float* src, int64_t d, int64_t lds, __nv
 size_t gram_tile_table_bytes(int64_t d);
 void gram_build_tiles(int64_t d, int2* tiles_host, int* lut_host, int* T_out);
 
-// CUDA-core kernels (kernels_simt.cu)
-cudaError_t launch_gram_simt(const void* V, int dtype, int64_t N, int64_t d, int64_t ld,
-                             const float* w, float scale, float* C, int64_t ldc, cudaStream_t s);
-cudaError_t launch_qform_simt(const void* V, int dtype, int64_t N, int64_t d, int64_t ld,
-                              const float* M, int64_t ldm, float* q, cudaStream_t s);
-cudaError_t launch_fwd_qform_simt(const void* V, int dtype, int64_t N, int64_t d, int64_t ld,
-                                  const float* F, int64_t ldf, float* q, cudaStream_t s);
+// small CUDA-core kernels (kernels_simt.cu)
 cudaError_t launch_rowsumsq(const void* V, int dtype, int64_t N, int64_t d, int64_t ld, float* q,
                             cudaStream_t s);
 cudaError_t launch_to_bf16(const float* src, int64_t rows, int64_t cols, int64_t lds,
                            __nv_bfloat16* dst, int64_t ldd, cudaStream_t s);
-// Cholesky L (lower, fp32), L^-1 (fp32, lower), logdet accumulated into st->logdet
-cudaError_t launch_cholesky(const float* F, int64_t d, int64_t ldf, float* L, float* Linv,
-                            float* work, float* diag_inv, DevStatus* st, int fault,
-                            cudaStream_t s);
-size_t cholesky_work_floats(int64_t d);
 // Streams and events of the look-ahead schedule of the tensor-core Cholesky: the panel
 // chain (diagonal block, panel solve, update of the next column block) runs on `crit`
 // (highest priority), the rest of each trailing update on `side` (lowest priority).

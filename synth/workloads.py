@@ -117,16 +117,31 @@ def exponent_for_condition(d: int, cond: float) -> float:
     return math.log(cond) / math.log(d) if d > 1 else 0.0
 
 
+_ORTHO_CACHE: dict = {}
+
+
 def orthogonal(d: int, gen: torch.Generator, device) -> torch.Tensor:
     """Seeded orthogonal d x d matrix (fp32): QR of a Gaussian matrix, signs fixed.
 
     The Gaussian matrix is drawn on the generator's device; the QR runs on the host in
-    fp64 (no device linear-algebra library is needed to draw inputs)."""
+    fp64 (no device linear-algebra library is needed to draw inputs).  A generator that
+    has drawn nothing yet always gives the same matrix, so those results are kept (the
+    large host QRs are then done once per process)."""
+    fresh = torch.Generator(device=gen.device)
+    fresh.manual_seed(gen.initial_seed())
+    key = (d, str(torch.device(device)), gen.initial_seed())
+    if torch.equal(gen.get_state(), fresh.get_state()) and key in _ORTHO_CACHE:
+        torch.randn(d, d, generator=gen, device=device, dtype=torch.float32)  # same draw
+        return _ORTHO_CACHE[key].to(device)
+    was_fresh = torch.equal(gen.get_state(), fresh.get_state())
     a = torch.randn(d, d, generator=gen, device=device, dtype=torch.float32)
     q, r = torch.linalg.qr(a.to("cpu", torch.float64))
     s = torch.sign(torch.diagonal(r))
     s[s == 0] = 1
-    return (q * s.unsqueeze(0)).to(device=device, dtype=torch.float32)
+    out = (q * s.unsqueeze(0)).to(torch.float32)
+    if was_fresh and d >= 1024:
+        _ORTHO_CACHE[key] = out
+    return out.to(device=device)
 
 
 def sqrt_cov(d: int, exponent: float, gen: torch.Generator, device) -> torch.Tensor:

@@ -22,7 +22,6 @@ import synth
 
 pytestmark = pytest.mark.gpu
 
-KERNELS = ["tc", "simt"]
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -42,16 +41,15 @@ def _bf16_gram_bound(V, w, scale):
 # ---------------------------------------------------------------------------
 # weighted Gram
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("kernel", KERNELS)
 @pytest.mark.parametrize("N,d,weighted", [(1000, 64, True), (5000, 320, True), (4097, 136, False),
                                           (3000, 512, True), (700, 8, True)])
-def test_weighted_gram_matches_oracle(kernel, N, d, weighted):
+def test_weighted_gram_matches_oracle(N, d, weighted):
     wl = synth.WORKLOADS["llama7b_attn_4096"].with_(n=d, m=8)
     X, _ = synth.rank_one_samples(wl, seed=1, device="cuda", N=N)
     w = (torch.rand(N, device="cuda", generator=torch.Generator("cuda").manual_seed(2)) * 3
          if weighted else None)
     scale = 1.0 / (N * 7)
-    with ffh.Handle(dtype="bf16", kernel=kernel) as h:
+    with ffh.Handle(dtype="bf16") as h:
         C = h.weighted_gram(X, w, scale)
     torch.cuda.synchronize()
     Vn = oracle.as_f64(X)
@@ -79,14 +77,13 @@ def test_weighted_gram_f32_input():
 # ---------------------------------------------------------------------------
 # quadratic form
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("kernel", KERNELS)
 @pytest.mark.parametrize("N,d", [(1000, 64), (3000, 264), (1500, 512), (129, 1024)])
-def test_quad_form_matches_oracle(kernel, N, d):
+def test_quad_form_matches_oracle(N, d):
     wl = synth.WORKLOADS["llama7b_attn_4096"].with_(n=d, m=8)
     X, _ = synth.rank_one_samples(wl, seed=4, device="cuda", N=N)
     A = oracle.as_f64(synth.spd_matrix(d, seed=5, cond=1e3, dtype=torch.float64))
     Linv = oracle.tri_inverse(oracle.cholesky(A))
-    with ffh.Handle(dtype="bf16", kernel=kernel) as h:
+    with ffh.Handle(dtype="bf16") as h:
         q = h.quad_form(X, torch.tensor(Linv, dtype=torch.float32, device="cuda"))
     Xn = oracle.as_f64(X)
     ref = oracle.inv_quad_forms_chol(oracle.cholesky(A), Xn)
@@ -101,30 +98,28 @@ def test_quad_form_matches_oracle(kernel, N, d):
 # ---------------------------------------------------------------------------
 # Cholesky and inverse
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("kernel", KERNELS)
 @pytest.mark.parametrize("d,cond", [(64, 1e2), (129, 1e2), (200, 1e3), (257, 1e3), (512, 1e3),
                                     (1000, 1e4), (1001, 1e3), (1536, 1e3), (2304, 1e3),
                                     (4096, 1e4)])
-def test_cholesky_matches_oracle(kernel, d, cond):
-    """Cholesky factor L and inverse M = L^-1.  Unit roundoff of the arithmetic:
-    CUDA-core path fp32 (u = 2^-24, accumulated over d terms); tensor-core path bf16
-    hi/lo split products (u = 2^-16 per product, fp32 accumulation).  Bounds: backward
+def test_cholesky_matches_oracle(d, cond):
+    """Cholesky factor L and inverse M = L^-1.  Unit roundoff of the arithmetic: bf16
+    hi/lo split products on the tensor cores (u = 2^-16 per product, fp32 accumulation).  Bounds: backward
     error ||L L^T - F|| / ||F|| <= 8 u_eff; inverse residual ||M L - I|| / sqrt(d) <=
     8 u_eff sqrt(cond); forward error of L <= 8 u_eff cond; log|F| to d u_eff cond."""
     A = synth.spd_matrix(d, seed=6, cond=cond, dtype=torch.float32, device="cuda")
-    with ffh.Handle(kernel=kernel) as h:
+    with ffh.Handle() as h:
         L, Li, logdet = h.cholesky(A)
     An = oracle.as_f64(A)
     Lr = oracle.cholesky(An)
     Mr = oracle.tri_inverse(Lr)
-    u_eff = 2.0 ** -16 if kernel == "tc" else d * 2.0 ** -24
+    u_eff = 2.0 ** -16
     Ln, Mn = oracle.as_f64(L), oracle.as_f64(Li)
     assert np.all(np.triu(Ln, 1) == 0) and np.all(np.triu(Mn, 1) == 0)
     back = np.linalg.norm(Ln @ Ln.T - An) / np.linalg.norm(An)
     inv_res = np.linalg.norm(Mn @ Ln - np.eye(d)) / math.sqrt(d)
     eL = np.linalg.norm(Ln - Lr) / np.linalg.norm(Lr)
     eM = np.linalg.norm(Mn - Mr) / np.linalg.norm(Mr)
-    print(f"d={d} cond={cond:g} {kernel}: back={back:.2e} inv={inv_res:.2e} eL={eL:.2e} "
+    print(f"d={d} cond={cond:g}: back={back:.2e} inv={inv_res:.2e} eL={eL:.2e} "
           f"eM={eM:.2e} dlogdet={abs(logdet - oracle.logdet_from_cholesky(Lr)):.2e}")
     assert back <= 8 * u_eff, back
     assert inv_res <= 8 * u_eff * math.sqrt(cond), inv_res
@@ -133,11 +128,10 @@ def test_cholesky_matches_oracle(kernel, d, cond):
     assert abs(logdet - oracle.logdet_from_cholesky(Lr)) <= d * u_eff * cond
 
 
-@pytest.mark.parametrize("kernel", KERNELS)
-def test_cholesky_rejects_indefinite(kernel):
+def test_cholesky_rejects_indefinite():
     A = torch.eye(300, device="cuda")
     A[150, 150] = -1.0
-    with ffh.Handle(kernel=kernel) as h:
+    with ffh.Handle() as h:
         with pytest.raises(ffh.FFHError) as ei:
             h.cholesky(A)
     assert ei.value.status == "FFH_ERR_NOT_SPD" and "150" in str(ei.value)
@@ -159,12 +153,11 @@ FIT_CASES = {
 }
 
 
-@pytest.mark.parametrize("kernel", KERNELS)
 @pytest.mark.parametrize("case", sorted(FIT_CASES))
-def test_fit_matches_oracle(case, kernel):
+def test_fit_matches_oracle(case):
     wl = FIT_CASES[case]
     X, G = synth.rank_one_samples(wl, seed=0, device="cuda")
-    with ffh.Handle(dtype=wl.dtype, kernel=kernel, final_loglik=True) as h:
+    with ffh.Handle(dtype=wl.dtype, final_loglik=True) as h:
         A, B = h.fit(X, G, iters=wl.iters)
         st = h.stats()
     ref = oracle.flipflop_fit(X.cpu(), G.cpu(), iters=wl.iters)
@@ -330,12 +323,11 @@ def test_fit_matrix_host_input_and_damping():
 # ---------------------------------------------------------------------------
 # Table 1 variants and the mismatch factor
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("kernel", KERNELS)
 @pytest.mark.parametrize("case", ["tiny_64", "llama_small"])
-def test_frobenius_fit_matches_oracle(case, kernel):
+def test_frobenius_fit_matches_oracle(case):
     wl = FIT_CASES[case].with_(iters=3)
     X, G = synth.rank_one_samples(wl, seed=0, device="cuda")
-    with ffh.Handle(dtype=wl.dtype, kernel=kernel, variant="frobenius") as h:
+    with ffh.Handle(dtype=wl.dtype, variant="frobenius") as h:
         A, B = h.fit(X, G, iters=wl.iters)
         st = h.stats()
     ref = oracle.frobenius_fit(X.cpu(), G.cpu(), iters=wl.iters)
