@@ -130,7 +130,9 @@ const char* ffh_last_error(ffh_t h);
  *   iters  maximum number of iterations (>= 1); one iteration = B-update, A-update
  *   tol    stop after iteration t when delta_t < tol, where
  *          delta_t = max_{F in {A,B}} ||F_t/tr F_t - F_{t-1}/tr F_{t-1}||_F / ||F_t/tr F_t||_F
- *          (delta_1 = +inf); tol = 0 runs exactly `iters` iterations
+ *          (delta_1 = +inf); tol = 0 runs exactly `iters` iterations.  The test runs on
+ *          the device: all `iters` iterations are enqueued, those after the stop return
+ *          at once, and the host synchronises once per call, at the end
  *   A_out  n x n fp32 (device or host): A with tr(A) = n
  *   B_out  m x m fp32 (device or host)
  * bf16 rows must be 16-byte aligned: n and m multiples of 8 for FFH_BF16 (fp32 inputs

@@ -8,11 +8,15 @@
 //   A_t = 1/(N m) X^T diag(r) X   (+ damping)
 //   s = tr(A_t)/n;  A_t /= s;  B_t *= s
 //   convergence statistics of A_t, B_t against A_{t-1}, B_{t-1}
-// all on the handle's stream; the host reads the device status once at the end (and
-// once per iteration only when tol > 0).
+// all on the handle's stream.  The stopping test runs on the device: a one-thread kernel
+// at the end of every iteration records the iteration and, when delta_t < tol, sets the
+// status block's `stop` word, after which the kernels of the remaining iterations (already
+// enqueued) return at once; the result is then copied from the slot of the last completed
+// iteration.  The host synchronises once per fit, at the end, to read the status.
 #include <stdarg.h>
 
 #include <cmath>
+#include <cstddef>
 #include <cstdio>
 #include <cstring>
 #include <string>
@@ -164,9 +168,10 @@ void prof_resolve(ffh_t h) {
   h->ev_used = 0;
 }
 
-ffh_status read_status(ffh_t h, DevStatus* st_dev) {
+ffh_status read_status(ffh_t h, DevStatus* st_dev, DevStatus* copy = nullptr) {
   DevStatus st;
   CK(cudaMemcpyAsync(&st, st_dev, sizeof(st), cudaMemcpyDeviceToHost, h->stream));
+  if (copy) *copy = st;
   CK(cudaStreamSynchronize(h->stream));
   prof_resolve(h);
   if (st.error == FFH_ERR_NOT_SPD)
@@ -395,7 +400,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
                     __nv_bfloat16** Gb, float** stage, float** q, float** r, float** A2,
                     float** B2, float** L, float** Linv, __nv_bfloat16** Mb, float** work,
                     int2** tn, int** ln, int2** tm, int** lm, float** partial,
-                    double** trb, __nv_bfloat16** Vw) {
+                    double** trb, __nv_bfloat16** Vw, float** Ares, float** Bres) {
     *st = c.take<DevStatus>(1);
     *recs = c.take<IterRecord>(iters + 2);
     const bool xcopy = dtype == FFH_F32 || (dtype == FFH_BF16 && !x_dev);
@@ -417,27 +422,31 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
     *tm = c.take<int2>(gram_tile_table_bytes(m) / sizeof(int2) + 1);
     *lm = c.take<int>(gram_tile_table_bytes(m) / sizeof(int) + 1);
     *partial = c.take<float>(std::max(gram_partial_bytes(pn), gram_partial_bytes(pm)) / 4);
-    *trb = c.take<double>(8);
+    *trb = c.take<double>(8 + kRedDoubles);  // statistics, then the reduction scratch
     *Vw = c.take<__nv_bfloat16>((size_t)N * pad8(D));
+    *Ares = c.take<float>((size_t)n * n);
+    *Bres = c.take<float>((size_t)m * m);
   };
   DevStatus* st;
   IterRecord* recs;
   __nv_bfloat16 *Xb, *Gb, *Mb, *Vw;
-  float *stage, *q, *r, *A2, *B2, *L, *Linv, *work, *partial;
+  float *stage, *q, *r, *A2, *B2, *L, *Linv, *work, *partial, *Ares, *Bres;
   int2 *tn, *tm;
   int *ln, *lm;
   double* trb;
   {
     Carve c(nullptr);
     layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &tn,
-           &ln, &tm, &lm, &partial, &trb, &Vw);
+           &ln, &tm, &lm, &partial, &trb, &Vw, &Ares, &Bres);
     ffh_status es = ensure_ws(h, c.off + 1024);
     if (es) return es;
   }
   Carve c(h->ws);
   layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &tn, &ln,
-         &tm, &lm, &partial, &trb, &Vw);
+         &tm, &lm, &partial, &trb, &Vw, &Ares, &Bres);
   cudaStream_t s = h->stream;
+  // the small kernels of this fit test its status block (see launch_iter_end)
+  GateScope gate(st);
   CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
   CK(cudaMemsetAsync(recs, 0, sizeof(IterRecord) * (iters + 2), s));
   CK(cudaMemsetAsync(q, 0, sizeof(float) * Npad, s));
@@ -471,7 +480,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
   const float sB = frob ? (float)(1.0 / (double)N) : (float)(1.0 / ((double)N * (double)n));
   const float sA = frob ? (float)(1.0 / (double)N) : (float)(1.0 / ((double)N * (double)m));
   int t_done = 0;
-  std::vector<IterRecord> host_recs((size_t)iters + 2);
+  std::vector<IterRecord> host_recs((size_t)std::max(iters, 1) + 2);
   if (variant == FFH_INPUT || variant == FFH_MARGINAL) {
     // Table 1: A = E[x x^T]; B = I (Input) or E[g g^T] (Marginal); then tr A = n
     const float s1 = (float)(1.0 / (double)N);
@@ -486,8 +495,8 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
     CK(launch_damp(A[cur], n, n, lam, st, s));
     CK(launch_damp(B[cur], m, m, lam, st, s));
     CK(launch_normalize(A[cur], n, B[cur], m, recs + 1, st, s));
+    CK(launch_iter_end(st, recs + 1, 1, 0.f, cur, s));
     iters = 0;  // no alternating loop
-    t_done = 1;
   }
   for (int t = 1; t <= iters; ++t) {
     IterRecord* R = recs + t;
@@ -503,77 +512,74 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
     } else {
       es = chol(h, A[cur], n, L, Linv, work, st, 0);
       if (es) return es;
-      CK(cudaMemcpyAsync(&R->logdet_A_prev, &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
-      if (t > 1)
-        CK(cudaMemcpyAsync(&recs[t - 1].logdet_A, &st->logdet, sizeof(double),
-                           cudaMemcpyDeviceToDevice, s));
+      CK(launch_copy_f64(&R->logdet_A_prev, &st->logdet, s));
+      if (t > 1) CK(launch_copy_f64(&recs[t - 1].logdet_A, &st->logdet, s));
       es = qform(h, xs, N, n, Linv, Mb, q, st);
       if (es) return es;
-      if (t > 1) CK(launch_dot(q, r, N, &recs[t - 1].sum_qr_A, s));
+      if (t > 1) CK(launch_dot(q, r, N, &recs[t - 1].sum_qr_A, trb + 8, s));
     }
     // ---- B-update
     es = gram(h, gs, N, m, q, sB, B[nxt], partial, gtm, st, Vw);
     if (es) return es;
     if (frob) {
-      CK(launch_frob2(A[cur], n, trb + 4, s));
+      CK(launch_frob2(A[cur], n, trb + 4, trb + 8, s));
       CK(launch_scale_by_inv(B[nxt], m, trb + 4, s));
     }
     CK(launch_damp(B[nxt], m, m, lam, st, s));
     es = chol(h, B[nxt], m, L, frob ? nullptr : Linv, work, st,
               (t == 1 && h->opt.fault == FFH_FAULT_BAD_PIVOT) ? FFH_FAULT_BAD_PIVOT : 0);
     if (es) return es;
-    CK(cudaMemcpyAsync(&R->logdet_B, &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
+    CK(launch_copy_f64(&R->logdet_B, &st->logdet, s));
     if (frob) {
       es = qform_fwd(h, gs, N, m, L, Mb, r, st);
     } else {
       es = qform(h, gs, N, m, Linv, Mb, r, st);
     }
     if (es) return es;
-    CK(launch_dot(q, r, N, &R->sum_qr_B, s));
+    CK(launch_dot(q, r, N, &R->sum_qr_B, trb + 8, s));
     // ---- A-update
     es = gram(h, xs, N, n, r, sA, A[nxt], partial, gtn, st, Vw);
     if (es) return es;
     if (frob) {
-      CK(launch_frob2(B[nxt], m, trb + 5, s));
+      CK(launch_frob2(B[nxt], m, trb + 5, trb + 8, s));
       CK(launch_scale_by_inv(A[nxt], n, trb + 5, s));
     }
     CK(launch_damp(A[nxt], n, n, lam, st, s));
     CK(launch_normalize(A[nxt], n, B[nxt], m, R, st, s));
-    // ---- convergence statistics
+    // ---- convergence statistics and the on-device stopping test
     CK(cudaMemsetAsync(&R->dA2, 0, sizeof(double) * 4, s));
     CK(launch_trace(A[nxt], n, trb + 0, s));
     CK(launch_trace(A[cur], n, trb + 1, s));
-    CK(launch_delta(A[nxt], A[cur], n, &R->dA2, &R->nA2, trb, s));
+    CK(launch_delta(A[nxt], A[cur], n, &R->dA2, &R->nA2, trb, trb + 8, s));
     if (t > 1) {
       CK(launch_trace(B[nxt], m, trb + 2, s));
       CK(launch_trace(B[cur], m, trb + 3, s));
-      CK(launch_delta(B[nxt], B[cur], m, &R->dB2, &R->nB2, trb + 2, s));
+      CK(launch_delta(B[nxt], B[cur], m, &R->dB2, &R->nB2, trb + 2, trb + 8, s));
     }
+    CK(launch_iter_end(st, R, t, tol, nxt, s));
     cur = nxt;
-    t_done = t;
-    if (tol > 0.f && t > 1) {
-      IterRecord hr;
-      CK(cudaMemcpyAsync(&hr, R, sizeof(hr), cudaMemcpyDeviceToHost, s));
-      CK(cudaStreamSynchronize(s));
-      const double dA = hr.nA2 > 0 ? std::sqrt(hr.dA2 / hr.nA2) : 0.0;
-      const double dB = hr.nB2 > 0 ? std::sqrt(hr.dB2 / hr.nB2) : 0.0;
-      if (std::max(dA, dB) < (double)tol) break;
-    }
   }
+  // the last completed iterate (the fit may have stopped before `iters`)
+  CK(launch_select_copy(st, A[0], A[1], Ares, n * n, s));
+  CK(launch_select_copy(st, B[0], B[1], Bres, m * m, s));
   if (h->opt.final_loglik && variant == FFH_FLIPFLOP) {
-    es = chol(h, A[cur], n, L, Linv, work, st, 0);
+    CK(launch_resume(st, s));
+    es = chol(h, Ares, n, L, Linv, work, st, 0);
     if (es) return es;
-    CK(cudaMemcpyAsync(&recs[t_done].logdet_A, &st->logdet, sizeof(double),
-                       cudaMemcpyDeviceToDevice, s));
+    CK(launch_record_at_done(st, recs, offsetof(IterRecord, logdet_A), &st->logdet, s));
     es = qform(h, xs, N, n, Linv, Mb, q, st);
     if (es) return es;
-    CK(launch_dot(q, r, N, &recs[t_done].sum_qr_A, s));
+    CK(launch_dot(q, r, N, trb + 6, trb + 8, s));
+    CK(launch_record_at_done(st, recs, offsetof(IterRecord, sum_qr_A), trb + 6, s));
   }
-  CK(cudaMemcpyAsync(A_out, A[cur], sizeof(float) * n * n, cudaMemcpyDefault, s));
-  CK(cudaMemcpyAsync(B_out, B[cur], sizeof(float) * m * m, cudaMemcpyDefault, s));
-  CK(cudaMemcpyAsync(host_recs.data(), recs, sizeof(IterRecord) * (iters + 2),
+  CK(cudaMemcpyAsync(A_out, Ares, sizeof(float) * n * n, cudaMemcpyDefault, s));
+  CK(cudaMemcpyAsync(B_out, Bres, sizeof(float) * m * m, cudaMemcpyDefault, s));
+  const int rec_count = std::max(iters, 1) + 2;
+  CK(cudaMemcpyAsync(host_recs.data(), recs, sizeof(IterRecord) * rec_count,
                      cudaMemcpyDeviceToHost, s));
-  es = read_status(h, st);
+  DevStatus hst;
+  es = read_status(h, st, &hst);
+  t_done = hst.iters_done;
   h->iters_done = t_done;
   h->N = N;
   h->n = n;
@@ -612,7 +618,7 @@ extern "C" ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_
                     float** stage, __nv_bfloat16** V, float** A2, float** B2, float** Cc,
                     float** L, float** Linv, __nv_bfloat16** Mb, float** work,
                     int2** tn, int** ln, int2** tm, int** lm, float** partial, double** trb,
-                    double** fro) {
+                    double** fro, float** Ares, float** Bres) {
     *st = c.take<DevStatus>(1);
     *recs = c.take<IterRecord>(iters + 2);
     *Gb = c.take<__nv_bfloat16>((size_t)N * mn);
@@ -630,27 +636,31 @@ extern "C" ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_
     *tm = c.take<int2>(gram_tile_table_bytes(m) / sizeof(int2) + 1);
     *lm = c.take<int>(gram_tile_table_bytes(m) / sizeof(int) + 1);
     *partial = c.take<float>(std::max(gram_partial_bytes(pa), gram_partial_bytes(pb)) / 4);
-    *trb = c.take<double>(8);
+    *trb = c.take<double>(8 + kRedDoubles);  // statistics, then the reduction scratch
     *fro = c.take<double>(4);
+    *Ares = c.take<float>((size_t)n * n);
+    *Bres = c.take<float>((size_t)m * m);
   };
   DevStatus* st;
   IterRecord* recs;
   __nv_bfloat16 *Gb, *V, *Mb;
-  float *stage, *A2, *B2, *Cc, *L, *Linv, *work, *partial;
+  float *stage, *A2, *B2, *Cc, *L, *Linv, *work, *partial, *Ares, *Bres;
   int2 *tn, *tm;
   int *ln, *lm;
   double *trb, *fro;
   {
     Carve c(nullptr);
     layout(c, &st, &recs, &Gb, &stage, &V, &A2, &B2, &Cc, &L, &Linv, &Mb, &work, &tn, &ln,
-           &tm, &lm, &partial, &trb, &fro);
+           &tm, &lm, &partial, &trb, &fro, &Ares, &Bres);
     ffh_status es = ensure_ws(h, c.off + 1024);
     if (es) return es;
   }
   Carve c(h->ws);
   layout(c, &st, &recs, &Gb, &stage, &V, &A2, &B2, &Cc, &L, &Linv, &Mb, &work, &tn, &ln, &tm,
-         &lm, &partial, &trb, &fro);
+         &lm, &partial, &trb, &fro, &Ares, &Bres);
   cudaStream_t s = h->stream;
+  // the small kernels of this fit test its status block (see launch_iter_end)
+  GateScope gate(st);
   CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
   CK(cudaMemsetAsync(recs, 0, sizeof(IterRecord) * (iters + 2), s));
   GramTables gtn, gtm;
@@ -687,7 +697,7 @@ extern "C" ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_
   auto half = [&](const __nv_bfloat16* Mbf, int64_t d, bool b_update, float scale, float* C,
                   const GramTables& gt) -> ffh_status {
     const int64_t d_other = b_update ? m : n;
-    CK(cudaMemsetAsync(C, 0, sizeof(float) * d_other * d_other, s));
+    CK(launch_zero_f32(C, d_other * d_other, st, s));
     for (int64_t k0 = 0; k0 < N; k0 += Kc) {
       const int64_t nk = std::min(Kc, N - k0);
       CK(launch_transform_tc(Mbf, d, d, Gb + k0 * mn, nk, m, n, b_update, V, st, s));
@@ -719,11 +729,10 @@ extern "C" ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_
     // ---- M_A = chol(A_{t-1})^-1 (bf16)
     es = chol(h, A[cur], n, L, Linv, work, st, 0);
     if (es) return es;
-    CK(cudaMemcpyAsync(&R->logdet_A_prev, &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
+    CK(launch_copy_f64(&R->logdet_A_prev, &st->logdet, s));
     if (t > 1) {
-      CK(cudaMemcpyAsync(&recs[t - 1].logdet_A, &st->logdet, sizeof(double),
-                         cudaMemcpyDeviceToDevice, s));
-      CK(launch_frob2(Linv, n, &recs[t - 1].trinvA, s));
+      CK(launch_copy_f64(&recs[t - 1].logdet_A, &st->logdet, s));
+      CK(launch_frob2(Linv, n, &recs[t - 1].trinvA, trb + 8, s));
     }
     CK(launch_lower_to_bf16(Linv, n, n, Mb, n, s));
     // ---- B-update
@@ -733,8 +742,8 @@ extern "C" ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_
     es = chol(h, B[nxt], m, L, Linv, work, st,
               (t == 1 && h->opt.fault == FFH_FAULT_BAD_PIVOT) ? FFH_FAULT_BAD_PIVOT : 0);
     if (es) return es;
-    CK(cudaMemcpyAsync(&R->logdet_B, &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
-    CK(launch_frob2(Linv, m, &R->trinvB, s));
+    CK(launch_copy_f64(&R->logdet_B, &st->logdet, s));
+    CK(launch_frob2(Linv, m, &R->trinvB, trb + 8, s));
     CK(launch_lower_to_bf16(Linv, m, m, Mb, m, s));
     // ---- A-update
     es = half(Mb, m, false, sA, A[nxt], gtn);
@@ -744,35 +753,33 @@ extern "C" ffh_status ffh_fit_matrix(ffh_t h, const float* Gk, int64_t N, int64_
     CK(cudaMemsetAsync(&R->dA2, 0, sizeof(double) * 4, s));
     CK(launch_trace(A[nxt], n, trb + 0, s));
     CK(launch_trace(A[cur], n, trb + 1, s));
-    CK(launch_delta(A[nxt], A[cur], n, &R->dA2, &R->nA2, trb, s));
+    CK(launch_delta(A[nxt], A[cur], n, &R->dA2, &R->nA2, trb, trb + 8, s));
     if (t > 1) {
       CK(launch_trace(B[nxt], m, trb + 2, s));
       CK(launch_trace(B[cur], m, trb + 3, s));
-      CK(launch_delta(B[nxt], B[cur], m, &R->dB2, &R->nB2, trb + 2, s));
+      CK(launch_delta(B[nxt], B[cur], m, &R->dB2, &R->nB2, trb + 2, trb + 8, s));
     }
+    CK(launch_iter_end(st, R, t, tol, nxt, s));
     cur = nxt;
-    t_done = t;
-    if (tol > 0.f && t > 1) {
-      IterRecord hr;
-      CK(cudaMemcpyAsync(&hr, R, sizeof(hr), cudaMemcpyDeviceToHost, s));
-      CK(cudaStreamSynchronize(s));
-      const double dA = hr.nA2 > 0 ? std::sqrt(hr.dA2 / hr.nA2) : 0.0;
-      const double dB = hr.nB2 > 0 ? std::sqrt(hr.dB2 / hr.nB2) : 0.0;
-      if (std::max(dA, dB) < (double)tol) break;
-    }
   }
+  // the last completed iterate (the fit may have stopped before `iters`)
+  CK(launch_select_copy(st, A[0], A[1], Ares, n * n, s));
+  CK(launch_select_copy(st, B[0], B[1], Bres, m * m, s));
   if (h->opt.final_loglik) {
-    es = chol(h, A[cur], n, L, Linv, work, st, 0);
+    CK(launch_resume(st, s));
+    es = chol(h, Ares, n, L, Linv, work, st, 0);
     if (es) return es;
-    CK(cudaMemcpyAsync(&recs[t_done].logdet_A, &st->logdet, sizeof(double),
-                       cudaMemcpyDeviceToDevice, s));
-    CK(launch_frob2(Linv, n, &recs[t_done].trinvA, s));
+    CK(launch_record_at_done(st, recs, offsetof(IterRecord, logdet_A), &st->logdet, s));
+    CK(launch_frob2(Linv, n, trb + 6, trb + 8, s));
+    CK(launch_record_at_done(st, recs, offsetof(IterRecord, trinvA), trb + 6, s));
   }
-  CK(cudaMemcpyAsync(A_out, A[cur], sizeof(float) * n * n, cudaMemcpyDefault, s));
-  CK(cudaMemcpyAsync(B_out, B[cur], sizeof(float) * m * m, cudaMemcpyDefault, s));
+  CK(cudaMemcpyAsync(A_out, Ares, sizeof(float) * n * n, cudaMemcpyDefault, s));
+  CK(cudaMemcpyAsync(B_out, Bres, sizeof(float) * m * m, cudaMemcpyDefault, s));
   CK(cudaMemcpyAsync(host_recs.data(), recs, sizeof(IterRecord) * (iters + 2),
                      cudaMemcpyDeviceToHost, s));
-  es = read_status(h, st);
+  DevStatus hst;
+  es = read_status(h, st, &hst);
+  t_done = hst.iters_done;
   // trace terms of the log-likelihood from exact identities:
   //   sum_k tr(B^-1 G_k A^-1 G_k^T) = N n tr(B^-1 S_B) = N n (m - shift_B tr(B^-1)) at the
   //   B-point (B = S_B + shift_B I), and N m (n - shift_A tr(A^-1)) at the A-point.
@@ -1104,7 +1111,7 @@ extern "C" ffh_status ffh_phi_tilde(ffh_t h, const void* X, const void* G, int64
     *Linv = c.take<float>((size_t)D * D);
     *Mb = c.take<__nv_bfloat16>((size_t)D * pad8(D));
     *work = c.take<float>(cholesky_tc_work_bytes(D) / 4 + 1);
-    *acc = c.take<double>(4);
+    *acc = c.take<double>(4 + kRedDoubles);  // results, then the reduction scratch
   };
   DevStatus* st;
   __nv_bfloat16 *Xb, *Gb, *Mb;
@@ -1136,7 +1143,7 @@ extern "C" ffh_status ffh_phi_tilde(ffh_t h, const void* X, const void* G, int64
   CK(cudaMemcpyAsync(&acc[2], &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
   es = qform(h, gs, N, m, Linv, Mb, r, st);
   if (es) return es;
-  CK(launch_dot(q, r, N, &acc[0], s));
+  CK(launch_dot(q, r, N, &acc[0], acc + 4, s));
   double hacc[3];
   CK(cudaMemcpyAsync(hacc, acc, sizeof(hacc), cudaMemcpyDeviceToHost, s));
   es = read_status(h, st);

@@ -48,9 +48,42 @@ struct DevStatus {
   int error;        // first FFH_ERR_* raised by a kernel (0 = none)
   int error_info;   // where: pivot index, or timeout site
   int abort_all;    // set together with error; kernels test it on entry
-  int pad;
+  int stop;         // the fit met its tolerance: the later iterations' kernels return at once
   double logdet;    // log|F| of the last Cholesky
   double acc[8];    // scratch reductions (traces, norms, dot products)
+  int iters_done;   // iterations completed (written by the end-of-iteration kernel)
+  int slot;         // ping-pong slot holding the last completed iterate (A and B)
+  int pad[2];
+};
+
+// true once a kernel raised an error or the fit stopped at its tolerance: the kernels of
+// a fit test this on entry (block-uniform) and return at once
+__device__ __forceinline__ bool halted(const DevStatus* st) {
+  return (*reinterpret_cast<const volatile int*>(&st->abort_all) |
+          *reinterpret_cast<const volatile int*>(&st->stop)) != 0;
+}
+// Block-uniform gate test for the entry of a kernel (every thread of the block must call
+// it): thread 0 reads the status and broadcasts it, so the block returns as a whole even
+// if another stream's kernel raises an error meanwhile.
+__device__ __forceinline__ bool gated_off(const DevStatus* gate) {
+  if (gate == nullptr) return false;
+  __shared__ int s_gated_off;
+  if (threadIdx.x == 0 && threadIdx.y == 0 && threadIdx.z == 0) s_gated_off = halted(gate) ? 1 : 0;
+  __syncthreads();
+  return s_gated_off != 0;
+}
+
+// The status block of the fit that is being enqueued by this host thread (a handle is
+// used by one thread at a time), or null.  Launchers of the small kernels pass it to
+// their kernels, which then do nothing once that fit has stopped or failed.  Set for the
+// duration of a fit by GateScope.
+const DevStatus* current_gate();
+void set_current_gate(const DevStatus* st);
+struct GateScope {
+  explicit GateScope(const DevStatus* st) { set_current_gate(st); }
+  ~GateScope() { set_current_gate(nullptr); }
+  GateScope(const GateScope&) = delete;
+  GateScope& operator=(const GateScope&) = delete;
 };
 
 // per-iteration record kept on the device, read once at the end of a fit
@@ -201,12 +234,31 @@ cudaError_t launch_transform_tc(const __nv_bfloat16* M, int64_t d, int64_t ldm,
 // A <- A / s, B <- B * s with s = tr(A)/n; records s and log-determinant corrections
 cudaError_t launch_normalize(float* A, int64_t n, float* B, int64_t m, IterRecord* rec,
                              DevStatus* st, cudaStream_t s);
+// fp64 reductions write per-block partial sums to a scratch of kRedDoubles doubles and add
+// them in a fixed order (bit-reproducible statistics)
+constexpr int kRedDoubles = 4096;
 cudaError_t launch_delta(const float* F, const float* Fprev, int64_t d, double* d2, double* n2,
-                         double* tr, cudaStream_t s);
-cudaError_t launch_dot(const float* a, const float* b, int64_t N, double* out, cudaStream_t s);
-cudaError_t launch_frob2(const float* F, int64_t d, double* out, cudaStream_t s);
+                         double* tr, double* red, cudaStream_t s);
+cudaError_t launch_dot(const float* a, const float* b, int64_t N, double* out, double* red,
+                       cudaStream_t s);
+cudaError_t launch_frob2(const float* F, int64_t d, double* out, double* red, cudaStream_t s);
 cudaError_t launch_scale_by_inv(float* F, int64_t d, const double* denom, cudaStream_t s);
-cudaError_t launch_copy_logdet(DevStatus* st, double* dst, cudaStream_t s);
-cudaError_t launch_zero_f64(double* p, int n, cudaStream_t s);
+// *dst = *src (fp64 record fields; gated like the other small kernels)
+cudaError_t launch_copy_f64(double* dst, const double* src, cudaStream_t s);
+// fp32 zero fill, skipped once `gate` has stopped or failed (gate may be null)
+cudaError_t launch_zero_f32(float* p, int64_t n, const DevStatus* gate, cudaStream_t s);
+// end of iteration t: unless the fit has stopped, record t and the slot of its iterate,
+// and with tol > 0 and t > 1 set st->stop when delta_t = max(sqrt(dA2/nA2),
+// sqrt(dB2/nB2)) of record R is below tol
+cudaError_t launch_iter_end(DevStatus* st, const IterRecord* R, int t, float tol, int slot,
+                            cudaStream_t s);
+// clear st->stop (the evaluation after a stopped fit runs again)
+cudaError_t launch_resume(DevStatus* st, cudaStream_t s);
+// dst = (st->slot ? src1 : src0), count floats
+cudaError_t launch_select_copy(const DevStatus* st, const float* src0, const float* src1,
+                               float* dst, int64_t count, cudaStream_t s);
+// recs[st->iters_done].<field at byte offset off> = *src
+cudaError_t launch_record_at_done(const DevStatus* st, IterRecord* recs, size_t off,
+                                  const double* src, cudaStream_t s);
 
 }  // namespace ffh

@@ -154,7 +154,7 @@ __global__ void __launch_bounds__(256, 1)
   volatile int* skip_flag = abort_flag + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    *skip_flag = *reinterpret_cast<volatile int*>(&a.st->abort_all);
+    *skip_flag = halted(a.st) ? 1 : 0;
     *abort_flag = 0;
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
@@ -520,7 +520,7 @@ __global__ void __launch_bounds__(256, 1)
   volatile int* skip_flag = abort_flag + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    *skip_flag = *reinterpret_cast<volatile int*>(&a.st->abort_all);
+    *skip_flag = halted(a.st) ? 1 : 0;
     *abort_flag = 0;
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
@@ -739,8 +739,10 @@ constexpr int SPLIT_TILE = 64;
 __global__ void __launch_bounds__(256) k_split_hilo(const float* __restrict__ src, int64_t lds,
                                                     int64_t src_stride, int rows, int cols,
                                                     int trans, __nv_bfloat16* __restrict__ dst,
-                                                    int rows_pad, int kpad) {
+                                                    int rows_pad, int kpad,
+                                                    const DevStatus* gate) {
   pdl_enter();
+  if (gated_off(gate)) return;
   __shared__ float tile[SPLIT_TILE][SPLIT_TILE + 1];
   const int z = blockIdx.z;
   const int r0 = blockIdx.y * SPLIT_TILE, c0 = blockIdx.x * SPLIT_TILE;
@@ -783,7 +785,7 @@ static cudaError_t split(const float* src, int64_t lds, int64_t src_stride, int 
   const dim3 grid((unsigned)(d.kpad / SPLIT_TILE), (unsigned)(d.rows_pad / SPLIT_TILE),
                   (unsigned)d.batch);
   cudaError_t e = launch_pdl(k_split_hilo, grid, dim3(256), 0, s, src, lds, src_stride, rows,
-                             cols, trans ? 1 : 0, d.p, d.rows_pad, d.kpad);
+                             cols, trans ? 1 : 0, d.p, d.rows_pad, d.kpad, current_gate());
   note_launches(1);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
@@ -1042,6 +1044,8 @@ __global__ void __launch_bounds__(LEAF_THREADS, 1) k_chol_leaf(float* W, int64_t
   float* T = sh + OFF_T;
   float* pivs = sh + OFF_PIV;
   pdl_enter();
+  // the fit this factorization belongs to has failed or stopped at its tolerance
+  if (gated_off(st)) return;
   const int b = (int)((d - o) < LB ? (d - o) : LB);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   // the lower triangle of the block, all loads of a thread in flight together

@@ -95,7 +95,7 @@ __global__ void __launch_bounds__(tf::THREADS, 1)
   volatile int* skip_flag = abort_flag + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    *skip_flag = *reinterpret_cast<volatile int*>(&a.st->abort_all);
+    *skip_flag = halted(a.st) ? 1 : 0;
     *abort_flag = 0;
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);

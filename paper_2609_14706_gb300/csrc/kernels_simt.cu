@@ -13,6 +13,10 @@ static std::atomic<long long> g_launches{0};
 void note_launches(int k) { g_launches.fetch_add(k, std::memory_order_relaxed); }
 long long launches_so_far() { return g_launches.load(std::memory_order_relaxed); }
 
+static thread_local const DevStatus* t_gate = nullptr;
+const DevStatus* current_gate() { return t_gate; }
+void set_current_gate(const DevStatus* st) { t_gate = st; }
+
 // SM count of the current device (cached per device; read and written atomically)
 int num_sms() {
   static std::atomic<int> cache[64];
@@ -94,7 +98,9 @@ cudaError_t launch_rowsumsq(const void* V, int dtype, int64_t N, int64_t d, int6
 // fp32 -> bf16 (pitch change, zero padding; `lower`: zero the strict upper triangle)
 // ---------------------------------------------------------------------------
 __global__ void k_to_bf16(const float* __restrict__ src, int64_t rows, int64_t cols, int64_t lds,
-                          __nv_bfloat16* __restrict__ dst, int64_t ldd, int lower) {
+                          __nv_bfloat16* __restrict__ dst, int64_t ldd, int lower,
+                          const DevStatus* gate) {
+  if (gated_off(gate)) return;
   const int64_t total = rows * ldd;
   for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
        idx += (int64_t)gridDim.x * blockDim.x) {
@@ -110,7 +116,9 @@ cudaError_t launch_to_bf16_ex(const float* src, int64_t rows, int64_t cols, int6
   const int64_t total = rows * ldd;
   if (total == 0) return cudaSuccess;
   const int64_t blocks = std::min<int64_t>((total + 255) / 256, (int64_t)num_sms() * 32);
-  k_to_bf16<<<(unsigned)blocks, 256, 0, s>>>(src, rows, cols, lds, dst, ldd, lower); note_launches(1);
+  k_to_bf16<<<(unsigned)blocks, 256, 0, s>>>(src, rows, cols, lds, dst, ldd, lower,
+                                               current_gate());
+  note_launches(1);
   return cudaGetLastError();
 }
 
@@ -127,7 +135,9 @@ cudaError_t launch_lower_to_bf16(const float* src, int64_t d, int64_t lds, __nv_
 // dst[r][c] = src[c][r] for c >= r (the transpose of a lower-triangular src), 0 below;
 // 32 x 32 tiles through shared memory
 __global__ void k_lowerT_to_bf16(const float* __restrict__ src, int64_t d, int64_t lds,
-                                 __nv_bfloat16* __restrict__ dst, int64_t ldd) {
+                                 __nv_bfloat16* __restrict__ dst, int64_t ldd,
+                                 const DevStatus* gate) {
+  if (gated_off(gate)) return;
   __shared__ float t[32][33];
   const int64_t bx = (int64_t)blockIdx.x * 32, by = (int64_t)blockIdx.y * 32;
   for (int r = threadIdx.y; r < 32; r += 8) {
@@ -146,7 +156,7 @@ __global__ void k_lowerT_to_bf16(const float* __restrict__ src, int64_t d, int64
 cudaError_t launch_lowerT_to_bf16(const float* src, int64_t d, int64_t lds, __nv_bfloat16* dst,
                                   int64_t ldd, cudaStream_t s) {
   const unsigned nb = (unsigned)((ldd + 31) / 32);
-  k_lowerT_to_bf16<<<dim3(nb, nb), dim3(32, 8), 0, s>>>(src, d, lds, dst, ldd);
+  k_lowerT_to_bf16<<<dim3(nb, nb), dim3(32, 8), 0, s>>>(src, d, lds, dst, ldd, current_gate());
   note_launches(1);
   return cudaGetLastError();
 }
@@ -171,7 +181,9 @@ cudaError_t launch_fill_identity(float* F, int64_t d, int64_t ld, cudaStream_t s
 
 // F += lambda * mean(diag F) * I (mean taken before the shift); the shift is also
 // written to *shift_out when given
-__global__ void k_damp(float* F, int64_t d, int64_t ld, float lambda, double* shift_out) {
+__global__ void k_damp(float* F, int64_t d, int64_t ld, float lambda, double* shift_out,
+                       const DevStatus* gate) {
+  if (gated_off(gate)) return;
   double acc = 0.0;
   for (int64_t i = threadIdx.x; i < d; i += blockDim.x) acc += F[i * ld + i];
   __shared__ double tot;
@@ -187,13 +199,14 @@ cudaError_t launch_damp(float* F, int64_t d, int64_t ld, float lambda, DevStatus
                         cudaStream_t s, double* shift_out) {
   if (lambda == 0.f) return shift_out ? cudaMemsetAsync(shift_out, 0, sizeof(double), s)
                                       : cudaSuccess;
-  k_damp<<<1, 1024, 0, s>>>(F, d, ld, lambda, shift_out);
+  k_damp<<<1, 1024, 0, s>>>(F, d, ld, lambda, shift_out, current_gate());
   note_launches(1);
   return cudaGetLastError();
 }
 
 // C += X (d x d, same pitch)
-__global__ void k_add(float* C, const float* X, int64_t total) {
+__global__ void k_add(float* C, const float* X, int64_t total, const DevStatus* gate) {
+  if (gated_off(gate)) return;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
        i += (int64_t)gridDim.x * blockDim.x)
     C[i] += X[i];
@@ -201,14 +214,15 @@ __global__ void k_add(float* C, const float* X, int64_t total) {
 
 cudaError_t launch_add(float* C, const float* X, int64_t total, cudaStream_t s) {
   const int64_t blocks = std::min<int64_t>((total + 255) / 256, (int64_t)num_sms() * 8);
-  k_add<<<(unsigned)std::max<int64_t>(1, blocks), 256, 0, s>>>(C, X, total);
+  k_add<<<(unsigned)std::max<int64_t>(1, blocks), 256, 0, s>>>(C, X, total, current_gate());
   note_launches(1);
   return cudaGetLastError();
 }
 
 // s = tr(A)/n, trB; stored into the record
 __global__ void k_norm_trace(const float* A, int64_t n, const float* B, int64_t m,
-                             IterRecord* rec) {
+                             IterRecord* rec, const DevStatus* gate) {
+  if (gated_off(gate)) return;
   double a = 0.0, b = 0.0;
   for (int64_t i = threadIdx.x; i < n; i += blockDim.x) a += A[i * n + i];
   for (int64_t i = threadIdx.x; i < m; i += blockDim.x) b += B[i * m + i];
@@ -222,7 +236,9 @@ __global__ void k_norm_trace(const float* A, int64_t n, const float* B, int64_t 
   }
 }
 
-__global__ void k_norm_apply(float* A, int64_t n, float* B, int64_t m, const IterRecord* rec) {
+__global__ void k_norm_apply(float* A, int64_t n, float* B, int64_t m, const IterRecord* rec,
+                             const DevStatus* gate) {
+  if (gated_off(gate)) return;
   const double sc = rec->scale;
   const float ia = (float)(1.0 / sc), sb = (float)sc;
   const int64_t tot_a = n * n, tot_b = m * m;
@@ -237,12 +253,13 @@ __global__ void k_norm_apply(float* A, int64_t n, float* B, int64_t m, const Ite
 
 cudaError_t launch_normalize(float* A, int64_t n, float* B, int64_t m, IterRecord* rec,
                              DevStatus*, cudaStream_t s) {
-  k_norm_trace<<<1, 1024, 0, s>>>(A, n, B, m, rec); note_launches(1);
+  k_norm_trace<<<1, 1024, 0, s>>>(A, n, B, m, rec, current_gate()); note_launches(1);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const int64_t tot = n * n + m * m;
   const int64_t blocks = std::min<int64_t>((tot + 255) / 256, (int64_t)num_sms() * 16);
-  k_norm_apply<<<(unsigned)blocks, 256, 0, s>>>(A, n, B, m, rec); note_launches(1);
+  k_norm_apply<<<(unsigned)blocks, 256, 0, s>>>(A, n, B, m, rec, current_gate());
+  note_launches(1);
   return cudaGetLastError();
 }
 
@@ -251,7 +268,8 @@ cudaError_t launch_normalize(float* A, int64_t n, float* B, int64_t m, IterRecor
 // the block and grid sums in fp64: FP64 arithmetic per element is slow on this part, and
 // the statistic needs only a few significant digits.
 __global__ void k_delta(const float* F, const float* P, int64_t total, const double* trF,
-                        const double* trP, double* d2, double* n2) {
+                        const double* trP, double* red, const DevStatus* gate) {
+  if (gated_off(gate)) return;
   const float a = (float)(1.0 / *trF), b = (float)(1.0 / *trP);
   float sdf = 0.f, snf = 0.f;
   const int64_t t0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -279,22 +297,52 @@ __global__ void k_delta(const float* F, const float* P, int64_t total, const dou
   __syncthreads();
   sn = block_sum_f64((double)snf);
   if (threadIdx.x == 0) {
-    atomicAdd(d2, sd);
-    atomicAdd(n2, sn);
+    red[2 * blockIdx.x] = sd;
+    red[2 * blockIdx.x + 1] = sn;
   }
 }
 
-cudaError_t launch_delta(const float* F, const float* Fprev, int64_t d, double* d2, double* n2,
-                         double* tr, cudaStream_t s) {
-  // tr[0] = tr(F), tr[1] = tr(Fprev)
-  const int64_t tot = d * d;
-  const int64_t blocks = std::min<int64_t>((tot + 255) / 256, (int64_t)num_sms() * 8);
-  k_delta<<<(unsigned)std::max<int64_t>(1, blocks), 256, 0, s>>>(F, Fprev, tot, tr, tr + 1, d2,
-                                                                  n2); note_launches(1);
+// out0 = sum_i red[nv i], out1 = sum_i red[nv i + 1] (nv = 1 or 2) over i < nb, in a fixed
+// order (one block: thread t adds partials t, t + 256, ... in turn, then a fixed tree), so
+// the fp64 statistics are the same on every run
+__global__ void k_sum_partials(const double* red, int nb, int nv, double* out0, double* out1,
+                               const DevStatus* gate) {
+  if (gated_off(gate)) return;
+  double a = 0.0, b = 0.0;
+  for (int i = threadIdx.x; i < nb; i += blockDim.x) {
+    a += red[(size_t)nv * i];
+    if (nv == 2) b += red[(size_t)nv * i + 1];
+  }
+  a = block_sum_f64(a);
+  __syncthreads();
+  b = block_sum_f64(b);
+  if (threadIdx.x == 0) {
+    *out0 = a;
+    if (out1) *out1 = b;
+  }
+}
+
+static cudaError_t sum_partials(const double* red, int nb, int nv, double* out0, double* out1,
+                                cudaStream_t s) {
+  k_sum_partials<<<1, 256, 0, s>>>(red, nb, nv, out0, out1, current_gate());
+  note_launches(1);
   return cudaGetLastError();
 }
 
-__global__ void k_trace_f64(const float* F, int64_t d, double* out) {
+cudaError_t launch_delta(const float* F, const float* Fprev, int64_t d, double* d2, double* n2,
+                         double* tr, double* red, cudaStream_t s) {
+  // tr[0] = tr(F), tr[1] = tr(Fprev)
+  const int64_t tot = d * d;
+  const int64_t blocks = std::max<int64_t>(
+      1, std::min<int64_t>({(tot + 255) / 256, (int64_t)num_sms() * 8, kRedDoubles / 2}));
+  k_delta<<<(unsigned)blocks, 256, 0, s>>>(F, Fprev, tot, tr, tr + 1, red, current_gate());
+  note_launches(1);
+  cudaError_t e = cudaGetLastError();
+  return e != cudaSuccess ? e : sum_partials(red, (int)blocks, 2, d2, n2, s);
+}
+
+__global__ void k_trace_f64(const float* F, int64_t d, double* out, const DevStatus* gate) {
+  if (gated_off(gate)) return;
   double a = 0.0;
   for (int64_t i = threadIdx.x; i < d; i += blockDim.x) a += F[i * d + i];
   a = block_sum_f64(a);
@@ -302,48 +350,56 @@ __global__ void k_trace_f64(const float* F, int64_t d, double* out) {
 }
 
 cudaError_t launch_trace(const float* F, int64_t d, double* out, cudaStream_t s) {
-  k_trace_f64<<<1, 1024, 0, s>>>(F, d, out); note_launches(1);
+  k_trace_f64<<<1, 1024, 0, s>>>(F, d, out, current_gate()); note_launches(1);
   return cudaGetLastError();
 }
 
-__global__ void k_dot(const float* a, const float* b, int64_t N, double* out) {
+__global__ void k_dot(const float* a, const float* b, int64_t N, double* red,
+                      const DevStatus* gate) {
+  if (gated_off(gate)) return;
   double acc = 0.0;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < N;
        i += (int64_t)gridDim.x * blockDim.x)
     acc += (double)a[i] * (double)b[i];
   acc = block_sum_f64(acc);
-  if (threadIdx.x == 0) atomicAdd(out, acc);
+  if (threadIdx.x == 0) red[blockIdx.x] = acc;
 }
 
-cudaError_t launch_dot(const float* a, const float* b, int64_t N, double* out, cudaStream_t s) {
-  cudaError_t e = cudaMemsetAsync(out, 0, sizeof(double), s);
-  if (e != cudaSuccess) return e;
-  const int64_t blocks = std::min<int64_t>((N + 255) / 256, (int64_t)num_sms() * 4);
-  k_dot<<<(unsigned)std::max<int64_t>(1, blocks), 256, 0, s>>>(a, b, N, out); note_launches(1);
-  return cudaGetLastError();
+cudaError_t launch_dot(const float* a, const float* b, int64_t N, double* out, double* red,
+                       cudaStream_t s) {
+  const int64_t blocks = std::max<int64_t>(
+      1, std::min<int64_t>({(N + 255) / 256, (int64_t)num_sms() * 4, kRedDoubles}));
+  k_dot<<<(unsigned)blocks, 256, 0, s>>>(a, b, N, red, current_gate());
+  note_launches(1);
+  cudaError_t e = cudaGetLastError();
+  return e != cudaSuccess ? e : sum_partials(red, (int)blocks, 1, out, nullptr, s);
 }
 
 // ||F||_F^2
-__global__ void k_frob2(const float* F, int64_t total, double* out) {
+__global__ void k_frob2(const float* F, int64_t total, double* red, const DevStatus* gate) {
+  if (gated_off(gate)) return;
   double acc = 0.0;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
        i += (int64_t)gridDim.x * blockDim.x)
     acc += (double)F[i] * (double)F[i];
   acc = block_sum_f64(acc);
-  if (threadIdx.x == 0) atomicAdd(out, acc);
+  if (threadIdx.x == 0) red[blockIdx.x] = acc;
 }
 
-cudaError_t launch_frob2(const float* F, int64_t d, double* out, cudaStream_t s) {
-  cudaError_t e = cudaMemsetAsync(out, 0, sizeof(double), s);
-  if (e != cudaSuccess) return e;
+cudaError_t launch_frob2(const float* F, int64_t d, double* out, double* red, cudaStream_t s) {
   const int64_t tot = d * d;
-  const int64_t blocks = std::min<int64_t>((tot + 255) / 256, (int64_t)num_sms() * 4);
-  k_frob2<<<(unsigned)std::max<int64_t>(1, blocks), 256, 0, s>>>(F, tot, out); note_launches(1);
-  return cudaGetLastError();
+  const int64_t blocks = std::max<int64_t>(
+      1, std::min<int64_t>({(tot + 255) / 256, (int64_t)num_sms() * 4, kRedDoubles}));
+  k_frob2<<<(unsigned)blocks, 256, 0, s>>>(F, tot, red, current_gate());
+  note_launches(1);
+  cudaError_t e = cudaGetLastError();
+  return e != cudaSuccess ? e : sum_partials(red, (int)blocks, 1, out, nullptr, s);
 }
 
 // F *= 1 / *denom
-__global__ void k_scale_by_inv(float* F, int64_t total, const double* denom) {
+__global__ void k_scale_by_inv(float* F, int64_t total, const double* denom,
+                               const DevStatus* gate) {
+  if (gated_off(gate)) return;
   const float f = (float)(1.0 / *denom);
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
        i += (int64_t)gridDim.x * blockDim.x)
@@ -353,7 +409,98 @@ __global__ void k_scale_by_inv(float* F, int64_t total, const double* denom) {
 cudaError_t launch_scale_by_inv(float* F, int64_t d, const double* denom, cudaStream_t s) {
   const int64_t tot = d * d;
   const int64_t blocks = std::min<int64_t>((tot + 255) / 256, (int64_t)num_sms() * 16);
-  k_scale_by_inv<<<(unsigned)std::max<int64_t>(1, blocks), 256, 0, s>>>(F, tot, denom); note_launches(1);
+  k_scale_by_inv<<<(unsigned)std::max<int64_t>(1, blocks), 256, 0, s>>>(F, tot, denom,
+                                                                         current_gate());
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// the on-device convergence test and the stopped-fit bookkeeping
+// ---------------------------------------------------------------------------
+__global__ void k_copy_f64(double* dst, const double* src, const DevStatus* gate) {
+  if (gated_off(gate)) return;
+  *dst = *src;
+}
+
+cudaError_t launch_copy_f64(double* dst, const double* src, cudaStream_t s) {
+  k_copy_f64<<<1, 1, 0, s>>>(dst, src, current_gate());
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+__global__ void k_zero_f32(float* p, int64_t n, const DevStatus* gate) {
+  if (gated_off(gate)) return;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    p[i] = 0.f;
+}
+
+cudaError_t launch_zero_f32(float* p, int64_t n, const DevStatus* gate, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  const int64_t blocks = std::min<int64_t>((n + 255) / 256, (int64_t)num_sms() * 4);
+  k_zero_f32<<<(unsigned)blocks, 256, 0, s>>>(p, n, gate);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+// One thread.  delta_t as in the fit's definition (Frobenius distance of the
+// trace-normalised iterates relative to the new one, the larger of A and B); the record
+// holds the squared distances and norms accumulated by k_delta.
+__global__ void k_iter_end(DevStatus* st, const IterRecord* R, int t, float tol, int slot) {
+  if (halted(st)) return;
+  st->iters_done = t;
+  st->slot = slot;
+  if (tol > 0.f && t > 1) {
+    const double dA = R->nA2 > 0.0 ? sqrt(R->dA2 / R->nA2) : 0.0;
+    const double dB = R->nB2 > 0.0 ? sqrt(R->dB2 / R->nB2) : 0.0;
+    if (fmax(dA, dB) < (double)tol) st->stop = 1;
+  }
+}
+
+cudaError_t launch_iter_end(DevStatus* st, const IterRecord* R, int t, float tol, int slot,
+                            cudaStream_t s) {
+  k_iter_end<<<1, 1, 0, s>>>(st, R, t, tol, slot);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+__global__ void k_resume(DevStatus* st) { st->stop = 0; }
+
+cudaError_t launch_resume(DevStatus* st, cudaStream_t s) {
+  k_resume<<<1, 1, 0, s>>>(st);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+__global__ void k_select_copy(const DevStatus* st, const float* __restrict__ src0,
+                              const float* __restrict__ src1, float* __restrict__ dst,
+                              int64_t count) {
+  const float* src = st->slot ? src1 : src0;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < count;
+       i += (int64_t)gridDim.x * blockDim.x)
+    dst[i] = src[i];
+}
+
+cudaError_t launch_select_copy(const DevStatus* st, const float* src0, const float* src1,
+                               float* dst, int64_t count, cudaStream_t s) {
+  if (count <= 0) return cudaSuccess;
+  const int64_t blocks = std::min<int64_t>((count + 255) / 256, (int64_t)num_sms() * 8);
+  k_select_copy<<<(unsigned)blocks, 256, 0, s>>>(st, src0, src1, dst, count);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+__global__ void k_record_at_done(const DevStatus* st, IterRecord* recs, size_t off,
+                                 const double* src) {
+  char* rec = reinterpret_cast<char*>(recs + st->iters_done);
+  *reinterpret_cast<double*>(rec + off) = *src;
+}
+
+cudaError_t launch_record_at_done(const DevStatus* st, IterRecord* recs, size_t off,
+                                  const double* src, cudaStream_t s) {
+  k_record_at_done<<<1, 1, 0, s>>>(st, recs, off, src);
+  note_launches(1);
   return cudaGetLastError();
 }
 

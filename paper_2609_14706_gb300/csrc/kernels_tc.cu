@@ -126,7 +126,7 @@ __global__ void __launch_bounds__(gram::THREADS, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    *skip_flag = *reinterpret_cast<volatile int*>(&a.st->abort_all);
+    *skip_flag = halted(a.st) ? 1 : 0;
     *abort_flag = 0;
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
@@ -327,10 +327,11 @@ __global__ void __launch_bounds__(gram::THREADS, 1)
 // write C[i][j] and C[j][i].  Block = 32 x 8 threads over one 32 x 32 block.
 __global__ void k_gram_reduce(const float* __restrict__ partial, const int* __restrict__ lut,
                               int nbn, int T, int S, int64_t d, float scale, float* C,
-                              int64_t ldc) {
+                              int64_t ldc, const DevStatus* gate) {
   using namespace gram;
   const int bi = blockIdx.y, bj = blockIdx.x;
   if (bj > bi) return;
+  if (gated_off(gate)) return;
   __shared__ float tile[32][33];
   const int64_t i0 = (int64_t)bi * 32, j0 = (int64_t)bj * 32;
   const size_t split_stride = (size_t)T * BN * BM;
@@ -439,7 +440,8 @@ cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t
   const int nb32 = (int)((d + 31) / 32);
   const int nbn = (int)((d + gram::BN - 1) / gram::BN);
   k_gram_reduce<<<dim3(nb32, nb32), dim3(32, 8), 0, s>>>(partial, lut_dev, nbn, plan.T, plan.S,
-                                                         d, scale, C, ldc); note_launches(1);
+                                                         d, scale, C, ldc, st);
+  note_launches(1);
   return cudaGetLastError();
 }
 
@@ -447,7 +449,8 @@ cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t
 // V^T diag(w) V); rounding as in the in-kernel scaling (fp32 product, one bf16 rounding).
 __global__ void k_scale_rows(const __nv_bfloat16* __restrict__ V, int64_t ld, int64_t N,
                              int64_t d8, const float* __restrict__ w, __nv_bfloat16* __restrict__ Vw,
-                             int64_t ldw) {
+                             int64_t ldw, const DevStatus* gate) {
+  if (gated_off(gate)) return;
   const int64_t total = N * d8;
   for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
        idx += (int64_t)gridDim.x * blockDim.x) {
@@ -472,7 +475,7 @@ cudaError_t launch_scale_rows(const __nv_bfloat16* V, int64_t ld, int64_t N, int
   const int64_t total = N * d8;
   if (total == 0) return cudaSuccess;
   const int64_t blocks = std::min<int64_t>((total + 255) / 256, (int64_t)num_sms() * 8);
-  k_scale_rows<<<(unsigned)blocks, 256, 0, s>>>(V, ld, N, d8, w, Vw, ldw);
+  k_scale_rows<<<(unsigned)blocks, 256, 0, s>>>(V, ld, N, d8, w, Vw, ldw, current_gate());
   note_launches(1);
   return cudaGetLastError();
 }
@@ -526,7 +529,7 @@ __global__ void __launch_bounds__(qf::THREADS, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    *skip_flag = *reinterpret_cast<volatile int*>(&a.st->abort_all);
+    *skip_flag = halted(a.st) ? 1 : 0;
     *abort_flag = 0;
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
@@ -714,7 +717,9 @@ cudaError_t launch_qform_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_
   a.st = st;
   a.budget_ns = kWaitBudgetNs;
   if (a.G == 2) {
-    cudaError_t e = cudaMemsetAsync(q, 0, sizeof(float) * N, s);
+    // two addends per entry: q starts at zero (skipped, like the kernel, once the fit
+    // has stopped, so the last completed pass's values stay)
+    cudaError_t e = launch_zero_f32(q, N, st, s);
     if (e != cudaSuccess) return e;
   }
   const int grid = std::min(a.RB * a.G, num_sms());

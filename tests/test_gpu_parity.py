@@ -23,7 +23,6 @@ import synth
 pytestmark = pytest.mark.gpu
 
 
-
 @pytest.fixture(scope="module", autouse=True)
 def _built():
     if not torch.cuda.is_available():
@@ -103,9 +102,10 @@ def test_quad_form_matches_oracle(N, d):
                                     (4096, 1e4)])
 def test_cholesky_matches_oracle(d, cond):
     """Cholesky factor L and inverse M = L^-1.  Unit roundoff of the arithmetic: bf16
-    hi/lo split products on the tensor cores (u = 2^-16 per product, fp32 accumulation).  Bounds: backward
-    error ||L L^T - F|| / ||F|| <= 8 u_eff; inverse residual ||M L - I|| / sqrt(d) <=
-    8 u_eff sqrt(cond); forward error of L <= 8 u_eff cond; log|F| to d u_eff cond."""
+    hi/lo split products on the tensor cores (u = 2^-16 per product, fp32 accumulation).
+    Bounds: backward error ||L L^T - F|| / ||F|| <= 8 u_eff; inverse residual
+    ||M L - I|| / sqrt(d) <= 8 u_eff sqrt(cond); forward error of L <= 8 u_eff cond;
+    log|F| to d u_eff cond."""
     A = synth.spd_matrix(d, seed=6, cond=cond, dtype=torch.float32, device="cuda")
     with ffh.Handle() as h:
         L, Li, logdet = h.cholesky(A)
@@ -215,6 +215,59 @@ def test_fit_tol_stops_early():
     ref = oracle.flipflop_fit(X.cpu(), G.cpu(), iters=50, tol=1e-4)
     assert st["iters_done"] < 50 and st["delta"] < 1e-4
     assert abs(st["iters_done"] - ref.iters_done) <= 1
+
+
+@pytest.mark.parametrize("case,tol", [("tiny_64", 1e-4), ("llama_small", 2e-3)])
+def test_stop_on_device_equals_fixed_count_fit(case, tol):
+    """The stopping test runs on the device: the fit enqueues all `iters` iterations and
+    the ones after delta_t < tol return at once.  The pair it returns, its statistics and
+    its final log-likelihood must be bit-identical to a fit of exactly iters_done
+    iterations (the fit is deterministic), and the skipped iterations must cost almost
+    nothing."""
+    wl = FIT_CASES[case]
+    X, G = synth.rank_one_samples(wl, seed=0, device="cuda")
+    with ffh.Handle(dtype=wl.dtype, final_loglik=True) as h:
+        A1, B1 = h.fit(X, G, iters=60, tol=tol)
+        st1 = h.stats()
+        T = st1["iters_done"]
+        assert 2 <= T < 60 and st1["delta"] < tol
+        A2, B2 = h.fit(X, G, iters=T)
+        st2 = h.stats()
+        # timing: 60 enqueued iterations that stop at T against T iterations
+        torch.cuda.synchronize()
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        e[0].record()
+        h.fit(X, G, iters=60, tol=tol)
+        e[1].record()
+        e[2].record()
+        h.fit(X, G, iters=T)
+        e[3].record()
+        torch.cuda.synchronize()
+    assert torch.equal(A1, A2) and torch.equal(B1, B2)
+    assert st2["iters_done"] == T
+    assert np.array_equal(np.array(st1["loglik"]), np.array(st2["loglik"]))
+    assert np.array_equal(np.array(st1["mean_qr"]), np.array(st2["mean_qr"]))
+    assert math.isfinite(st1["loglik"][-1])
+    t_stop, t_fixed = e[0].elapsed_time(e[1]), e[2].elapsed_time(e[3])
+    print(f"\n{case}: stopped at {T} of 60; {t_stop:.2f} ms vs {t_fixed:.2f} ms for {T} iterations")
+    # each skipped iteration is a few dozen launches that return at once
+    assert t_stop < t_fixed + (60 - T) * 1.0 + 5.0
+
+
+def test_stop_on_device_matrix_fit():
+    wl = synth.WORKLOADS["kron_recovery_512x768"].with_(n=64, m=96)
+    Gk = synth.matrix_samples(wl, seed=3, device="cuda", N=256)
+    with ffh.Handle(dtype="f32", final_loglik=True) as h:
+        A1, B1 = h.fit_matrix(Gk, 40, 1e-4)
+        st1 = h.stats()
+        T = st1["iters_done"]
+        A2, B2 = h.fit_matrix(Gk, T, 0.0)
+        st2 = h.stats()
+    assert 2 <= T < 40
+    assert torch.equal(A1, A2) and torch.equal(B1, B2)
+    assert np.array_equal(np.array(st1["loglik"]), np.array(st2["loglik"]))
+    ref = oracle.flipflop_fit_matrix(Gk.cpu(), iters=40, tol=1e-4)
+    assert abs(T - ref.iters_done) <= 1
 
 
 def test_fit_warm_start():
