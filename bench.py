@@ -71,12 +71,12 @@ def measured_peaks():
 
 def gram_source_sha256() -> str:
     """sha256 of the Gram kernel's source: kernels_tc.cu from `namespace gram {` up to the
-    scaling pass that follows the Gram launcher (kernel, tile tables, reduction, launch)."""
+    quadratic-form section (kernel, tile tables, reduction, launch)."""
     src = os.path.join(ROOT, "paper_2609_14706_gb300", "csrc", "kernels_tc.cu")
     with open(src) as f:
         text = f.read()
     a = text.index("namespace gram {")
-    b = text.index("__global__ void k_scale_rows")
+    b = text.index("// fused quadratic form")
     return hashlib.sha256(text[a:b].encode()).hexdigest()
 
 
@@ -348,7 +348,8 @@ def run_ours(args):
     qform_flops_step = 0.0 if matrix else iters * (ffh.qform_flops(N, n) + ffh.qform_flops(N, m))
     qform_tflops = ((qform_flops_step * args.steps) / (tim["qform_ms"] / 1e3) / 1e12
                     if tim["qform_ms"] > 0 else None)
-    roofline = {"bound": "tensor", "kernel": "k_gram_tc (weighted Gram)",
+    roofline = {"bound": "tensor",
+                "kernel": "k_gram_tc (weighted Gram, diag(w) applied in its operand load)",
                 "achieved": gram_tflops, "peak": peak, "unit": "TFLOP/s",
                 "frac": gram_tflops / peak, "traffic": profiled_traffic(wl.name),
                 "traffic_unit": "bytes per launch (ncu dram__bytes_read + write)",

@@ -296,23 +296,14 @@ ffh_status stage_input(ffh_t h, const void* V, bool on_dev, int64_t N, int64_t d
   return FFH_OK;
 }
 
-// C = scale * V^T diag(w) V.  With a scratch `vw` (N rows of V.ld_bf bf16) the weights are
-// applied to a copy of V first and the tensor-core Gram runs unweighted on (diag(w) V, V):
-// the same bf16 operands, without the in-kernel scaling pass competing with the MMA for
-// shared-memory bandwidth.
+// C = scale * V^T diag(w) V on the tensor cores; the weights enter the kernel's operand
+// load (no scaled copy of V).
 ffh_status gram(ffh_t h, const Staged& V, int64_t N, int64_t d, const float* w_padded, float scale,
-                float* C, float* partial, const GramTables& gt, DevStatus* st,
-                __nv_bfloat16* vw = nullptr) {
+                float* C, float* partial, const GramTables& gt, DevStatus* st) {
   cudaEvent_t t0 = prof_begin(h);
   cudaEvent_t t1 = t0 ? next_event(h) : nullptr;
-  const __nv_bfloat16* va = nullptr;
-  if (vw && w_padded) {
-    CK(launch_scale_rows(V.bf, V.ld_bf, N, d, w_padded, vw, V.ld_bf, h->stream));
-    va = vw;
-    w_padded = nullptr;
-  }
   CK(launch_gram_tc(V.bf, N, d, V.ld_bf, w_padded, scale, C, d, partial, gt.tiles, gt.lut,
-                    gt.plan, st, h->opt.fault, h->stream, t1, va, V.ld_bf));
+                    gt.plan, st, h->opt.fault, h->stream, t1));
   prof_end(h, PROF_GRAM, t0, t1);
   return FFH_OK;
 }
@@ -400,7 +391,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
                     __nv_bfloat16** Gb, float** stage, float** q, float** r, float** A2,
                     float** B2, float** L, float** Linv, __nv_bfloat16** Mb, float** work,
                     int2** tn, int** ln, int2** tm, int** lm, float** partial,
-                    double** trb, __nv_bfloat16** Vw, float** Ares, float** Bres) {
+                    double** trb, float** Ares, float** Bres) {
     *st = c.take<DevStatus>(1);
     *recs = c.take<IterRecord>(iters + 2);
     const bool xcopy = dtype == FFH_F32 || (dtype == FFH_BF16 && !x_dev);
@@ -423,13 +414,12 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
     *lm = c.take<int>(gram_tile_table_bytes(m) / sizeof(int) + 1);
     *partial = c.take<float>(std::max(gram_partial_bytes(pn), gram_partial_bytes(pm)) / 4);
     *trb = c.take<double>(8 + kRedDoubles);  // statistics, then the reduction scratch
-    *Vw = c.take<__nv_bfloat16>((size_t)N * pad8(D));
     *Ares = c.take<float>((size_t)n * n);
     *Bres = c.take<float>((size_t)m * m);
   };
   DevStatus* st;
   IterRecord* recs;
-  __nv_bfloat16 *Xb, *Gb, *Mb, *Vw;
+  __nv_bfloat16 *Xb, *Gb, *Mb;
   float *stage, *q, *r, *A2, *B2, *L, *Linv, *work, *partial, *Ares, *Bres;
   int2 *tn, *tm;
   int *ln, *lm;
@@ -437,13 +427,13 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
   {
     Carve c(nullptr);
     layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &tn,
-           &ln, &tm, &lm, &partial, &trb, &Vw, &Ares, &Bres);
+           &ln, &tm, &lm, &partial, &trb, &Ares, &Bres);
     ffh_status es = ensure_ws(h, c.off + 1024);
     if (es) return es;
   }
   Carve c(h->ws);
   layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &tn, &ln,
-         &tm, &lm, &partial, &trb, &Vw, &Ares, &Bres);
+         &tm, &lm, &partial, &trb, &Ares, &Bres);
   cudaStream_t s = h->stream;
   // the small kernels of this fit test its status block (see launch_iter_end)
   GateScope gate(st);
@@ -519,7 +509,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
       if (t > 1) CK(launch_dot(q, r, N, &recs[t - 1].sum_qr_A, trb + 8, s));
     }
     // ---- B-update
-    es = gram(h, gs, N, m, q, sB, B[nxt], partial, gtm, st, Vw);
+    es = gram(h, gs, N, m, q, sB, B[nxt], partial, gtm, st);
     if (es) return es;
     if (frob) {
       CK(launch_frob2(A[cur], n, trb + 4, trb + 8, s));
@@ -538,7 +528,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
     if (es) return es;
     CK(launch_dot(q, r, N, &R->sum_qr_B, trb + 8, s));
     // ---- A-update
-    es = gram(h, xs, N, n, r, sA, A[nxt], partial, gtn, st, Vw);
+    es = gram(h, xs, N, n, r, sA, A[nxt], partial, gtn, st);
     if (es) return es;
     if (frob) {
       CK(launch_frob2(B[nxt], m, trb + 5, trb + 8, s));

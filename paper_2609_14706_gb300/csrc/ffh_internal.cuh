@@ -170,18 +170,14 @@ struct GramPlan {
 GramPlan gram_plan(int64_t N, int64_t d, int sms);
 size_t gram_partial_bytes(const GramPlan& p);
 // C = scale * V^T diag(w) V (lower tiles, then mirrored), V bf16 N x d (pitch ld elements).
-// With Va (pitch lda) the A operand is read from Va instead of V: C = scale * Va^T V, for
-// Va = diag(w) V pre-scaled by launch_scale_rows (then w_padded must be null).
+// w_padded (nullable: w = 1) must be readable up to KB * kGramBK entries, zero past N; with
+// weights, d and ld are multiples of 8 and V is 16-byte aligned.  after_main, if given, is
+// recorded between the main kernel and the reduction.
 cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t ld,
                            const float* w_padded, float scale, float* C, int64_t ldc,
                            float* partial, int2* tiles_dev, int* tile_lut_dev,
                            const GramPlan& plan, DevStatus* st, int fault, cudaStream_t s,
-                           cudaEvent_t after_main = nullptr, const __nv_bfloat16* Va = nullptr,
-                           int64_t lda = 0);
-// Vw[k][:] = bf16(w_k V[k][:]), bf16 rows of d elements (pitches multiples of 8 elements,
-// 16-byte aligned; the padding up to the next multiple of 8 is written too)
-cudaError_t launch_scale_rows(const __nv_bfloat16* V, int64_t ld, int64_t N, int64_t d,
-                              const float* w, __nv_bfloat16* Vw, int64_t ldw, cudaStream_t s);
+                           cudaEvent_t after_main = nullptr);
 // q_k = ||M v_k||^2, V bf16 N x d (pitch ld), M bf16 d x d lower (pitch ldm)
 cudaError_t launch_qform_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t ld,
                             const __nv_bfloat16* M, int64_t ldm, float* q, DevStatus* st,

@@ -5,11 +5,12 @@
 //                   so both MMA operands are the same V read "MN-major": TMA boxes of
 //                   64 features x 64 samples, 128-byte swizzle.  diag(w) is applied to the
 //                   A operand in shared memory between the TMA landing and the MMA (one
-//                   16-byte vector = 8 features of one sample share one weight).  Only the
-//                   tiles that meet the lower triangle are computed; K (samples) is split
-//                   into S slices so that tiles x slices fill the SMs; fp32 partial tiles
-//                   go to a workspace and k_gram_reduce sums them in a fixed order,
-//                   applies the scale and writes both triangles.
+//                   16-byte vector = 8 features of one sample share one weight), so no
+//                   scaled copy of V exists anywhere.  Only the tiles that meet the lower
+//                   triangle are computed; K (samples) is split into S slices so that
+//                   tiles x slices fill the SMs; fp32 partial tiles go to a workspace and
+//                   k_gram_reduce sums them in a fixed order, applies the scale and writes
+//                   both triangles.
 //  * k_qform_tc  -- q_k = ||M v_k||^2 for lower-triangular M = L^-1 (the x^T A^-1 x of
 //                   Section 5).  Y = V M^T is formed tile by tile in TMEM and squared and
 //                   row-summed by the epilogue straight from TMEM, so Y never reaches
@@ -406,17 +407,12 @@ size_t gram_partial_bytes(const GramPlan& p) {
 cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t ld,
                            const float* w_padded, float scale, float* C, int64_t ldc,
                            float* partial, int2* tiles_dev, int* lut_dev, const GramPlan& plan,
-                           DevStatus* st, int fault, cudaStream_t s, cudaEvent_t after_main,
-                           const __nv_bfloat16* Va, int64_t lda) {
-  CUtensorMap bmap, amap;
-  if (!make_map_bf16(&bmap, V, (uint64_t)d, (uint64_t)N, (uint64_t)ld, 64, gram::BK))
+                           DevStatus* st, int fault, cudaStream_t s, cudaEvent_t after_main) {
+  // the weights are bulk-copied 64 at a time (16-byte aligned source)
+  if (w_padded && (reinterpret_cast<uintptr_t>(w_padded) & 15)) return cudaErrorInvalidValue;
+  CUtensorMap map;
+  if (!make_map_bf16(&map, V, (uint64_t)d, (uint64_t)N, (uint64_t)ld, 64, gram::BK))
     return cudaErrorInvalidValue;
-  if (Va && w_padded) return cudaErrorInvalidValue;  // a pre-scaled A operand carries the weights
-  if (!Va) {
-    amap = bmap;
-  } else if (!make_map_bf16(&amap, Va, (uint64_t)d, (uint64_t)N, (uint64_t)lda, 64, gram::BK)) {
-    return cudaErrorInvalidValue;
-  }
   static PerDeviceOnce attr;
   {
     cudaError_t e = smem_attr_once((const void*)k_gram_tc, gram::SMEM_BYTES, attr);
@@ -433,7 +429,8 @@ cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t
   a.st = st;
   a.fault = fault;
   a.budget_ns = fault == FFH_FAULT_LOST_COPY ? kFaultWaitBudgetNs : kWaitBudgetNs;
-  k_gram_tc<<<plan.grid, gram::THREADS, gram::SMEM_BYTES, s>>>(amap, bmap, a); note_launches(1);
+  k_gram_tc<<<plan.grid, gram::THREADS, gram::SMEM_BYTES, s>>>(map, map, a);
+  note_launches(1);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   if (after_main && (e = cudaEventRecord(after_main, s)) != cudaSuccess) return e;
@@ -441,41 +438,6 @@ cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t
   const int nbn = (int)((d + gram::BN - 1) / gram::BN);
   k_gram_reduce<<<dim3(nb32, nb32), dim3(32, 8), 0, s>>>(partial, lut_dev, nbn, plan.T, plan.S,
                                                          d, scale, C, ldc, st);
-  note_launches(1);
-  return cudaGetLastError();
-}
-
-// Vw[k][:] = bf16(w_k V[k][:]) (the A operand of an unweighted Gram that equals
-// V^T diag(w) V); rounding as in the in-kernel scaling (fp32 product, one bf16 rounding).
-__global__ void k_scale_rows(const __nv_bfloat16* __restrict__ V, int64_t ld, int64_t N,
-                             int64_t d8, const float* __restrict__ w, __nv_bfloat16* __restrict__ Vw,
-                             int64_t ldw, const DevStatus* gate) {
-  if (gated_off(gate)) return;
-  const int64_t total = N * d8;
-  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
-       idx += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t row = idx / d8, c = idx - row * d8;
-    const float s = w[row];
-    uint4 v = *reinterpret_cast<const uint4*>(V + row * ld + 8 * c);
-    v.x = scale_bf16x2(v.x, s);
-    v.y = scale_bf16x2(v.y, s);
-    v.z = scale_bf16x2(v.z, s);
-    v.w = scale_bf16x2(v.w, s);
-    *reinterpret_cast<uint4*>(Vw + row * ldw + 8 * c) = v;
-  }
-}
-
-cudaError_t launch_scale_rows(const __nv_bfloat16* V, int64_t ld, int64_t N, int64_t d,
-                              const float* w, __nv_bfloat16* Vw, int64_t ldw, cudaStream_t s) {
-  // rows are processed in 8-element chunks up to the padded width (the pitches are
-  // multiples of 8); the padding columns are never read as operands
-  if (ld % 8 || ldw % 8 || ((reinterpret_cast<uintptr_t>(V) | reinterpret_cast<uintptr_t>(Vw)) & 15))
-    return cudaErrorInvalidValue;
-  const int64_t d8 = (d + 7) / 8;
-  const int64_t total = N * d8;
-  if (total == 0) return cudaSuccess;
-  const int64_t blocks = std::min<int64_t>((total + 255) / 256, (int64_t)num_sms() * 8);
-  k_scale_rows<<<(unsigned)blocks, 256, 0, s>>>(V, ld, N, d8, w, Vw, ldw, current_gate());
   note_launches(1);
   return cudaGetLastError();
 }
