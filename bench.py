@@ -13,7 +13,9 @@ flush is needed between steps.
                   [--workload NAME] [--samples N]
 
 With N > 1 (torchrun, one rank per GPU) every rank fits its own layer (independent
-problems, weak scaling, no collective in the data path); rank 0 prints the line.
+problems, weak scaling, no collective in the data path); rank 0 prints the line.  With
+--sharded the ranks instead fit one layer together: rank r holds N / world of its samples
+and the partial Grams of every half-step are summed over ranks with NCCL (strong scaling).
 --impl reference times the fp64 CPU oracle on a bounded sample of the same workload.
 """
 from __future__ import annotations
@@ -54,6 +56,8 @@ def parse_args():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-waterkron", action="store_true",
                    help="skip the WaterKron quantizer timing on the fitted factors")
+    p.add_argument("--sharded", action="store_true",
+                   help="one layer fitted by all ranks together, samples split over ranks")
     p.add_argument("--samples", type=int, default=None,
                    help="override the workload's sample count N (short profiling runs; "
                         "the headline uses the workload's own N)")
@@ -265,6 +269,10 @@ def run_ours(args):
     matrix = wl.kind == "matrix"
     iters = wl.iters
     N, n, m = wl.N, wl.n, wl.m
+    if args.sharded:
+        if matrix:
+            raise SystemExit("--sharded: rank-one workloads only")
+        return run_sharded(args, wl, rank, world, dist)
     # each rank fits its own layer (independent problems)
     if matrix:
         Gk = synth.matrix_samples(wl, seed=args.seed + rank, device="cuda")
@@ -419,6 +427,54 @@ def run_ours(args):
         "roofline": roofline, "kernels": kernels, "waterkron": waterkron, "cpu_baseline": cpu,
         "e2e": e2e,
         "gpu_launches": int(launches), "clocks": clk,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    h.close()
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def run_sharded(args, wl, rank, world, dist):
+    """One layer fitted by all ranks: rank r draws its own N / world samples (seed + r) and
+    the partial Grams are summed over ranks every half-step (fit_sharded)."""
+    from paper_2609_14706_gb300.sharded import fit_sharded
+
+    n_local = wl.N // world + (1 if rank < wl.N % world else 0)
+    X, G = synth.rank_one_samples(wl, seed=args.seed + rank, device="cuda", N=n_local)
+    reduce = (lambda t: dist.all_reduce(t)) if dist is not None else None
+    import paper_2609_14706_gb300 as ffh
+
+    h = ffh.Handle(dtype=wl.dtype)
+    for _ in range(max(args.warmup, 3)):
+        fit_sharded([(X, G)], wl.iters, reduce_sum=reduce, n_total=wl.N, handle=h)
+    stream = torch.cuda.current_stream()
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    barrier()
+    clocks = ClockSampler(int(os.environ.get("LOCAL_RANK", "0")))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        fit_sharded([(X, G)], wl.iters, reduce_sum=reduce, n_total=wl.N, handle=h)
+    e1.record(stream)
+    barrier()
+    clk = clocks.stop()
+    elapsed_ms = max_over_ranks(e0.elapsed_time(e1), dist, "cuda")
+    value = args.steps * wl.iters / (elapsed_ms / 1e3)   # iterations of the one shared fit
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
+        "scaling": "strong", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": wl.name, "N": wl.N, "n": wl.n, "m": wl.m,
+                   "iters_per_step": wl.iters, "parallelism": f"samples sharded over {world}",
+                   "l2": "inputs exceed L2; no flush"},
+        "gpu_launches": None, "clocks": clk,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)

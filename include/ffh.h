@@ -201,6 +201,44 @@ ffh_status ffh_quad_form(ffh_t h, const void* V, const float* Linv, int64_t N, i
 ffh_status ffh_cholesky(ffh_t h, const float* F, int64_t d, float* L_out, float* Linv_out,
                         double* logdet);
 
+/* ---- sample-sharded fit (device pointers; handle's stream) ----
+ * Every update of Section 5 is an expectation, i.e. a sum over the N samples, so ranks
+ * that hold disjoint shards of the samples can each form the unscaled partial sum of
+ * their shard, add the partial sums over all ranks (the caller's all-reduce, e.g. NCCL),
+ * and finish the update identically on every rank.  One half-step (the B-update shown;
+ * the A-update swaps the roles of X and G):
+ *   ffh_partial_gram(h, X_r, G_r, N_r, n, m, A, P)   on each rank r
+ *   all-reduce P (sum over ranks)
+ *   ffh_update_from_sum(h, P, m, 1 / (N n), B)       N = sum_r N_r
+ * then ffh_normalize_pair after the A-update and ffh_relative_change for the stop test.
+ * The Python driver fit_sharded (package paper_2609_14706_gb300.sharded) composes them. */
+
+/* P = sum_k w_k v_k v_k^T over the N rows of this shard, unscaled, with
+ * w_k = u_k^T F^-1 u_k (F = NULL: w_k = ||u_k||^2, i.e. F = I, the first B-update):
+ *   U          N x du samples whose quadratic forms weight the sum (X for the B-update)
+ *   V          N x dv samples of the Gram (G for the B-update); U, V dtype opt.dtype
+ *   F          du x du fp32 SPD, or NULL
+ *   accumulate 0: P_out = P;  1: P_out += P (a process holding several shards)
+ *   P_out      dv x dv fp32, full symmetric
+ *   logdet_F   host double, log|F| (0 for F = NULL); nullable
+ * Errors: INVALID_ARG, NOT_SPD, OOM, CUDA, TIMEOUT. */
+ffh_status ffh_partial_gram(ffh_t h, const void* U, const void* V, int64_t N, int64_t du,
+                            int64_t dv, const float* F, int32_t accumulate, float* P_out,
+                            double* logdet_F);
+
+/* F_out = scale * P, then the handle's damping F += lambda mean(diag F) I (Appendix B):
+ * the update from the partial sums added over all ranks (scale = 1/(N d_other)).
+ * P, F_out: d x d fp32 (may alias).  Errors: INVALID_ARG, CUDA. */
+ffh_status ffh_update_from_sum(ffh_t h, const float* P, int64_t d, double scale, float* F_out);
+
+/* s = tr(A)/n; A <- A / s; B <- B * s (the scale freedom of Section 5); s_out nullable. */
+ffh_status ffh_normalize_pair(ffh_t h, float* A, int64_t n, float* B, int64_t m, double* s_out);
+
+/* delta = ||F/tr F - Fprev/tr Fprev||_F / ||F/tr F||_F (the fit's stopping statistic for
+ * one factor); delta_out: host double. */
+ffh_status ffh_relative_change(ffh_t h, const float* F, const float* Fprev, int64_t d,
+                               double* delta_out);
+
 /* ---- WaterKron downstream of the fit (Sections 2-3; device pointers, handle's stream) ---- */
 
 /* Reverse Cholesky (Section 2 notation: RevCholesky(F) is the lower L with L_ii > 0 and

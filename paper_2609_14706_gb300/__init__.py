@@ -89,6 +89,10 @@ def load_library(path: Optional[str] = None):
         "ffh_rev_cholesky": ([vp, vp, i64, vp, vp, pd], ctypes.c_int),
         "ffh_waterfilling_scales": ([vp, vp, i64, vp, i64, f32, vp, vp], ctypes.c_int),
         "ffh_gptq2": ([vp, vp, vp, vp, vp, vp, i64, i64, vp, vp], ctypes.c_int),
+        "ffh_partial_gram": ([vp, vp, vp, i64, i64, i64, vp, i32, vp, pd], ctypes.c_int),
+        "ffh_update_from_sum": ([vp, vp, i64, ctypes.c_double, vp], ctypes.c_int),
+        "ffh_normalize_pair": ([vp, vp, i64, vp, i64, pd], ctypes.c_int),
+        "ffh_relative_change": ([vp, vp, vp, i64, pd], ctypes.c_int),
     }
     for name, (args, res) in sigs.items():
         fn = getattr(lib, name)
@@ -282,6 +286,53 @@ class Handle:
         code = self._lib.ffh_cholesky(self._h, _ptr(F), d, _ptr(L), _ptr(Li), ctypes.byref(ld))
         _check(self._lib, self._h, code, "ffh_cholesky")
         return L, Li, ld.value
+
+    # ---- sample-sharded fit steps ----
+    def partial_gram(self, U: torch.Tensor, V: torch.Tensor, F: Optional[torch.Tensor],
+                     P_out: Optional[torch.Tensor] = None, accumulate: bool = False):
+        """ffh_partial_gram: (P = sum_k (u_k^T F^-1 u_k) v_k v_k^T over these rows, log|F|);
+        F None means F = I; accumulate adds P into P_out."""
+        U, V = self._samples(U, "U"), self._samples(V, "V")
+        N, du = U.shape
+        dv = V.shape[1]
+        if F is not None:
+            F = F.to(torch.float32).contiguous()
+        if P_out is None:
+            if accumulate:
+                raise ValueError("accumulate needs P_out")
+            P_out = torch.empty(dv, dv, dtype=torch.float32, device=V.device)
+        ld = ctypes.c_double()
+        code = self._lib.ffh_partial_gram(self._h, _ptr(U), _ptr(V), N, du, dv, _ptr(F),
+                                          int(bool(accumulate)), _ptr(P_out), ctypes.byref(ld))
+        _check(self._lib, self._h, code, "ffh_partial_gram")
+        return P_out, ld.value
+
+    def update_from_sum(self, P: torch.Tensor, scale: float,
+                        F_out: Optional[torch.Tensor] = None) -> torch.Tensor:
+        """ffh_update_from_sum: damp(scale * P) with the handle's damping."""
+        P = P.contiguous()
+        if F_out is None:
+            F_out = torch.empty_like(P)
+        code = self._lib.ffh_update_from_sum(self._h, _ptr(P), P.shape[0], float(scale),
+                                             _ptr(F_out))
+        _check(self._lib, self._h, code, "ffh_update_from_sum")
+        return F_out
+
+    def normalize_pair(self, A: torch.Tensor, B: torch.Tensor) -> float:
+        """ffh_normalize_pair: A /= s, B *= s with s = tr(A)/n (in place); returns s."""
+        out = ctypes.c_double()
+        code = self._lib.ffh_normalize_pair(self._h, _ptr(A), A.shape[0], _ptr(B), B.shape[0],
+                                            ctypes.byref(out))
+        _check(self._lib, self._h, code, "ffh_normalize_pair")
+        return out.value
+
+    def relative_change(self, F: torch.Tensor, Fprev: torch.Tensor) -> float:
+        """ffh_relative_change: ||F/trF - P/trP||_F / ||F/trF||_F."""
+        out = ctypes.c_double()
+        code = self._lib.ffh_relative_change(self._h, _ptr(F), _ptr(Fprev), F.shape[0],
+                                             ctypes.byref(out))
+        _check(self._lib, self._h, code, "ffh_relative_change")
+        return out.value
 
     # ---- WaterKron downstream (Sections 2-3) ----
     def rev_cholesky(self, F: torch.Tensor):

@@ -1144,3 +1144,167 @@ extern "C" ffh_status ffh_phi_tilde(ffh_t h, const void* X, const void* G, int64
                       std::log(mean_qr / ((double)m * (double)n)));
   return FFH_OK;
 }
+
+// ---------------------------------------------------------------------------
+// sample-sharded fit: the steps a driver composes around a sum over ranks
+// ---------------------------------------------------------------------------
+extern "C" ffh_status ffh_partial_gram(ffh_t h, const void* U, const void* V, int64_t N,
+                                       int64_t du, int64_t dv, const float* F,
+                                       int32_t accumulate, float* P_out, double* logdet_F) {
+  if (!h) return FFH_ERR_INVALID_ARG;
+  h->err.clear();
+  ffh_status vs = validate_opt(h);
+  if (vs) return vs;
+  if (!U || !V || !P_out || N < 1 || du < 1 || dv < 1)
+    return fail(h, FFH_ERR_INVALID_ARG, "bad arguments");
+  if (N > (int64_t)1 << 30) return fail(h, FFH_ERR_INVALID_ARG, "N too large");
+  if (!is_device_ptr(U) || !is_device_ptr(V) || !is_device_ptr(P_out) || (F && !is_device_ptr(F)))
+    return fail(h, FFH_ERR_INVALID_ARG, "ffh_partial_gram takes device pointers");
+  const int dtype = h->opt.dtype;
+  if (dtype == FFH_BF16 && (du % 8 || dv % 8))
+    return fail(h, FFH_ERR_INVALID_ARG, "bf16 rows must be 16-byte aligned: du, dv multiples of 8");
+  const int64_t Npad = (N + 63) / 64 * 64 + 64;
+  GramPlan plan = gram_plan(N, dv, num_sms());
+  auto layout = [&](Carve& c, DevStatus** st, __nv_bfloat16** Ub, __nv_bfloat16** Vb, float** w,
+                    float** L, float** Linv, __nv_bfloat16** Mb, float** work, float** partial,
+                    int2** tiles, int** lut, float** Ptmp) {
+    *st = c.take<DevStatus>(1);
+    *Ub = (dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(du)) : nullptr;
+    *Vb = (dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(dv)) : nullptr;
+    *w = c.take<float>(Npad);
+    *L = F ? c.take<float>((size_t)du * du) : nullptr;
+    *Linv = F ? c.take<float>((size_t)du * du) : nullptr;
+    *Mb = F ? c.take<__nv_bfloat16>((size_t)du * pad8(du)) : nullptr;
+    *work = F ? c.take<float>(cholesky_tc_work_bytes(du) / 4 + 1) : nullptr;
+    *partial = c.take<float>(gram_partial_bytes(plan) / 4);
+    *tiles = c.take<int2>(gram_tile_table_bytes(dv) / sizeof(int2) + 1);
+    *lut = c.take<int>(gram_tile_table_bytes(dv) / sizeof(int) + 1);
+    *Ptmp = accumulate ? c.take<float>((size_t)dv * dv) : nullptr;
+  };
+  DevStatus* st;
+  __nv_bfloat16 *Ub, *Vb, *Mb;
+  float *w, *L, *Linv, *work, *partial, *Ptmp;
+  int2* tiles;
+  int* lut;
+  {
+    Carve c(nullptr);
+    layout(c, &st, &Ub, &Vb, &w, &L, &Linv, &Mb, &work, &partial, &tiles, &lut, &Ptmp);
+    ffh_status es = ensure_ws(h, c.off + 1024);
+    if (es) return es;
+  }
+  Carve c(h->ws);
+  layout(c, &st, &Ub, &Vb, &w, &L, &Linv, &Mb, &work, &partial, &tiles, &lut, &Ptmp);
+  cudaStream_t s = h->stream;
+  CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
+  CK(cudaMemsetAsync(w, 0, sizeof(float) * Npad, s));
+  Staged us, vs_;
+  ffh_status es = stage_input(h, U, true, N, du, Ub, nullptr, &us);
+  if (es) return es;
+  es = stage_input(h, V, true, N, dv, Vb, nullptr, &vs_);
+  if (es) return es;
+  // weights w_k = u_k^T F^-1 u_k (F = I: ||u_k||^2)
+  if (F) {
+    es = chol(h, F, du, L, Linv, work, st, 0);
+    if (es) return es;
+    es = qform(h, us, N, du, Linv, Mb, w, st);
+    if (es) return es;
+  } else {
+    CK(launch_rowsumsq(us.raw, dtype, N, du, us.ld_raw, w, s));
+  }
+  GramTables gt;
+  es = setup_tables(h, N, dv, &gt, tiles, lut);
+  if (es) return es;
+  es = gram(h, vs_, N, dv, w, 1.0f, accumulate ? Ptmp : P_out, partial, gt, st);
+  if (es) return es;
+  if (accumulate) CK(launch_add(P_out, Ptmp, dv * dv, s));
+  DevStatus hst;
+  es = read_status(h, st, &hst);
+  if (logdet_F) *logdet_F = F ? hst.logdet : 0.0;
+  return es;
+}
+
+extern "C" ffh_status ffh_update_from_sum(ffh_t h, const float* P, int64_t d, double scale,
+                                          float* F_out) {
+  if (!h) return FFH_ERR_INVALID_ARG;
+  h->err.clear();
+  ffh_status vs = validate_opt(h);
+  if (vs) return vs;
+  if (!P || !F_out || d < 1 || !(scale > 0.0) || !std::isfinite(scale))
+    return fail(h, FFH_ERR_INVALID_ARG, "bad arguments");
+  if (!is_device_ptr(P) || !is_device_ptr(F_out))
+    return fail(h, FFH_ERR_INVALID_ARG, "ffh_update_from_sum takes device pointers");
+  DevStatus* st;
+  {
+    Carve c(nullptr);
+    c.take<DevStatus>(1);
+    ffh_status es = ensure_ws(h, c.off + 1024);
+    if (es) return es;
+  }
+  Carve c(h->ws);
+  st = c.take<DevStatus>(1);
+  cudaStream_t s = h->stream;
+  CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
+  CK(launch_scale_copy(P, F_out, d * d, scale, s));
+  CK(launch_damp(F_out, d, d, h->opt.damping, st, s));
+  return read_status(h, st);
+}
+
+extern "C" ffh_status ffh_normalize_pair(ffh_t h, float* A, int64_t n, float* B, int64_t m,
+                                         double* s_out) {
+  if (!h) return FFH_ERR_INVALID_ARG;
+  h->err.clear();
+  if (!A || !B || n < 1 || m < 1) return fail(h, FFH_ERR_INVALID_ARG, "bad arguments");
+  if (!is_device_ptr(A) || !is_device_ptr(B))
+    return fail(h, FFH_ERR_INVALID_ARG, "ffh_normalize_pair takes device pointers");
+  DevStatus* st;
+  IterRecord* rec;
+  {
+    Carve c(nullptr);
+    c.take<DevStatus>(1);
+    c.take<IterRecord>(1);
+    ffh_status es = ensure_ws(h, c.off + 1024);
+    if (es) return es;
+  }
+  Carve c(h->ws);
+  st = c.take<DevStatus>(1);
+  rec = c.take<IterRecord>(1);
+  cudaStream_t s = h->stream;
+  CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
+  CK(launch_normalize(A, n, B, m, rec, st, s));
+  IterRecord hr;
+  CK(cudaMemcpyAsync(&hr, rec, sizeof(hr), cudaMemcpyDeviceToHost, s));
+  ffh_status es = read_status(h, st);
+  if (s_out) *s_out = hr.scale;
+  return es;
+}
+
+extern "C" ffh_status ffh_relative_change(ffh_t h, const float* F, const float* Fprev, int64_t d,
+                                          double* delta_out) {
+  if (!h) return FFH_ERR_INVALID_ARG;
+  h->err.clear();
+  if (!F || !Fprev || !delta_out || d < 1) return fail(h, FFH_ERR_INVALID_ARG, "bad arguments");
+  if (!is_device_ptr(F) || !is_device_ptr(Fprev))
+    return fail(h, FFH_ERR_INVALID_ARG, "ffh_relative_change takes device pointers");
+  DevStatus* st;
+  double* acc;
+  {
+    Carve c(nullptr);
+    c.take<DevStatus>(1);
+    c.take<double>(4 + kRedDoubles);
+    ffh_status es = ensure_ws(h, c.off + 1024);
+    if (es) return es;
+  }
+  Carve c(h->ws);
+  st = c.take<DevStatus>(1);
+  acc = c.take<double>(4 + kRedDoubles);  // tr F, tr Fprev, d2, n2, then the scratch
+  cudaStream_t s = h->stream;
+  CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
+  CK(launch_trace(F, d, acc + 0, s));
+  CK(launch_trace(Fprev, d, acc + 1, s));
+  CK(launch_delta(F, Fprev, d, acc + 2, acc + 3, acc, acc + 4, s));
+  double hacc[4];
+  CK(cudaMemcpyAsync(hacc, acc, sizeof(hacc), cudaMemcpyDeviceToHost, s));
+  ffh_status es = read_status(h, st);
+  *delta_out = hacc[3] > 0 ? std::sqrt(hacc[2] / hacc[3]) : 0.0;
+  return es;
+}

@@ -239,6 +239,9 @@ cudaError_t launch_dot(const float* a, const float* b, int64_t N, double* out, d
                        cudaStream_t s);
 cudaError_t launch_frob2(const float* F, int64_t d, double* out, double* red, cudaStream_t s);
 cudaError_t launch_scale_by_inv(float* F, int64_t d, const double* denom, cudaStream_t s);
+// dst = scale * src
+cudaError_t launch_scale_copy(const float* src, float* dst, int64_t count, double scale,
+                              cudaStream_t s);
 // *dst = *src (fp64 record fields; gated like the other small kernels)
 cudaError_t launch_copy_f64(double* dst, const double* src, cudaStream_t s);
 // fp32 zero fill, skipped once `gate` has stopped or failed (gate may be null)

@@ -504,4 +504,22 @@ cudaError_t launch_record_at_done(const DevStatus* st, IterRecord* recs, size_t 
   return cudaGetLastError();
 }
 
+// dst = scale * src (count floats; the product in fp64, one rounding)
+__global__ void k_scale_copy(const float* __restrict__ src, float* __restrict__ dst,
+                             int64_t count, double scale, const DevStatus* gate) {
+  if (gated_off(gate)) return;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < count;
+       i += (int64_t)gridDim.x * blockDim.x)
+    dst[i] = (float)((double)src[i] * scale);
+}
+
+cudaError_t launch_scale_copy(const float* src, float* dst, int64_t count, double scale,
+                              cudaStream_t s) {
+  if (count <= 0) return cudaSuccess;
+  const int64_t blocks = std::min<int64_t>((count + 255) / 256, (int64_t)num_sms() * 8);
+  k_scale_copy<<<(unsigned)blocks, 256, 0, s>>>(src, dst, count, scale, current_gate());
+  note_launches(1);
+  return cudaGetLastError();
+}
+
 }  // namespace ffh
