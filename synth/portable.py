@@ -8,15 +8,18 @@ same samples, so this module draws them in a way that does not depend on the mac
 * every normal variate comes from numpy's PCG64 generator (integer state), seeded by a
   SeedSequence of (seed, stream[, chunk]), in fp64, one generator per fixed chunk of
   rows, so the bytes do not depend on how many threads draw them;
-* the mixing x = S z and every scaling are done in fp64, on the host or on a GPU;
-* the result is rounded once to fp32 and then, for bf16 workloads, to bf16 (both
-  round-to-nearest-even).
+* the mixing x = S z is exact in fp64: z is put on a grid of 2^-8 (clipped to |z| <= 8)
+  and S on a grid of 2^-26 (|S_ij| <= 1), so every product is an integer multiple of
+  2^-34 below 2^37 of those units and every partial sum of up to 2^14 of them stays
+  below 2^51 < 2^53: any order of the additions (another BLAS, a GPU) gives the same
+  result, bit for bit;
+* the remaining steps (the Student-t factor, outlier and g scales) are single IEEE
+  operations per element, and the result is rounded once to fp32 and then, for bf16
+  workloads, to bf16 (both round-to-nearest-even).
 
-fp64 arithmetic done in another order (another BLAS, a GPU's) moves a value by a few
-units in its last place; that changes the rounded value only when the value lies that
-close to a rounding midpoint, about once in 10^13 bf16 elements (10^8 for fp32
-elements).  ``sha256`` digests the bytes so that both sides can confirm they saw the
-same samples.
+The grids are far finer than anything the statistics of a fit can see (the normal
+variate moves by at most 2^-9, an entry of S by 2^-27).  ``sha256`` digests the bytes so
+that both sides can confirm they saw the same samples.
 
 The recipe is the one of ``workloads.py`` (power-law covariances with a Haar-like
 rotation, outlier channels, multivariate Student-t inputs, g scale); only the random
@@ -36,6 +39,11 @@ from .workloads import Workload, exponent_for_condition
 
 # rows per generator chunk; fixed, so the bytes never depend on memory or threads
 CHUNK_ROWS = 8192
+# the exact-mixing grids: z in 2^-Z_BITS units (|z| <= Z_CLIP), S in 2^-S_BITS units
+Z_BITS, Z_CLIP, S_BITS = 8, 8.0, 26
+# matrix samples: the intermediate S_B Z_k is put on a 2^-Y_BITS grid (|.| <= Y_CLIP) and
+# S_A on a 2^-SA_BITS grid, so the second product is exact as well (512 terms)
+Y_BITS, Y_CLIP, SA_BITS = 12, 1024.0, 20
 
 # stream keys (a namespace of their own: 1000 + k)
 _QX, _QG, _ZX, _ZG, _OUT, _W, _QA, _QB, _ZK = (1000 + k for k in range(9))
@@ -55,10 +63,23 @@ def orthogonal64(d: int, seed: int, stream: int) -> np.ndarray:
     return q * s[None, :]
 
 
-def sqrt_cov64(d: int, exponent: float, seed: int, stream: int) -> np.ndarray:
-    """S = Q diag(lambda)^{1/2} (fp64), lambda_i = i^-exponent, so S S^T = Q diag(lambda) Q^T."""
+def _grid(a: np.ndarray, bits: int, clip: float = None) -> np.ndarray:
+    """Nearest multiple of 2^-bits (ties to even; exact in fp64 for |a| < 2^(53 - bits))."""
+    if clip is not None:
+        a = np.clip(a, -clip, clip)
+    return np.rint(a * (2.0 ** bits)) * (2.0 ** -bits)
+
+
+def sqrt_cov64(d: int, exponent: float, seed: int, stream: int, bits: int = S_BITS) -> np.ndarray:
+    """S = Q diag(lambda)^{1/2} (fp64), lambda_i = i^-exponent, so S S^T = Q diag(lambda) Q^T,
+    on the 2^-bits grid (|S_ij| <= 1, since lambda_i <= 1 and Q is orthogonal)."""
     lam = np.arange(1, d + 1, dtype=np.float64) ** (-float(exponent))
-    return orthogonal64(d, seed, stream) * np.sqrt(lam)[None, :]
+    return _grid(orthogonal64(d, seed, stream) * np.sqrt(lam)[None, :], bits)
+
+
+def _normals(seed: int, key: int, c: int, shape) -> np.ndarray:
+    """Standard normal variates on the 2^-Z_BITS grid, clipped to |z| <= Z_CLIP."""
+    return _grid(_rng(seed, key, c).standard_normal(shape), Z_BITS, Z_CLIP)
 
 
 def _threads() -> int:
@@ -79,7 +100,8 @@ def rank_one_samples(wl: Workload, seed: int = 0, device="cpu", N: Optional[int]
 
     x_k = S_x z_k (Gaussian) or S_x z_k / sqrt(w_k / nu) (multivariate Student-t,
     w_k a sum of nu squared normals), then the outlier channels are scaled;
-    g_k = g_scale S_g z'_k.  All of it in fp64, one rounding at the end."""
+    g_k = g_scale S_g z'_k.  The mixing is exact, the rest single IEEE fp64 operations,
+    one rounding at the end."""
     assert wl.kind == "rank_one"
     N = wl.N if N is None else int(N)
     dev = torch.device(device)
@@ -96,8 +118,8 @@ def rank_one_samples(wl: Workload, seed: int = 0, device="cpu", N: Optional[int]
     def draw(c: int):
         r0 = c * CHUNK_ROWS
         rows = min(N, r0 + CHUNK_ROWS) - r0
-        zx = _rng(seed, _ZX, c).standard_normal((rows, wl.n))
-        zg = _rng(seed, _ZG, c).standard_normal((rows, wl.m))
+        zx = _normals(seed, _ZX, c, (rows, wl.n))
+        zg = _normals(seed, _ZG, c, (rows, wl.m))
         f = None
         if nu:
             u = _rng(seed, _W, c).standard_normal((rows, nu))
@@ -129,8 +151,9 @@ def rank_one_samples(wl: Workload, seed: int = 0, device="cpu", N: Optional[int]
 
 def matrix_normal_factors(wl: Workload, seed: int = 0):
     """(S_A, S_B) in fp64 on the host for the matrix workload: S S^T = A0 (n x n), B0
-    (m x m), power-law spectra with condition number wl.cond."""
-    SA = sqrt_cov64(wl.n, exponent_for_condition(wl.n, wl.cond), seed, _QA)
+    (m x m), power-law spectra with condition number wl.cond (S_A on the coarser grid
+    of the second, exact, product)."""
+    SA = sqrt_cov64(wl.n, exponent_for_condition(wl.n, wl.cond), seed, _QA, bits=SA_BITS)
     SB = sqrt_cov64(wl.m, exponent_for_condition(wl.m, wl.cond), seed, _QB)
     return SA, SB
 
@@ -138,8 +161,10 @@ def matrix_normal_factors(wl: Workload, seed: int = 0):
 def matrix_sample_chunk(wl: Workload, seed: int, k0: int, k1: int, SA_t: torch.Tensor,
                         SB_t: torch.Tensor) -> torch.Tensor:
     """Samples k0..k1-1 of the matrix workload, G_k = S_B Z_k S_A^T (fp64 on the device
-    of SA_t, rounded once to wl.dtype).  Samples are drawn per generator chunk of
-    CHUNK_ROWS // 64 samples, so any k0..k1 reproduce the same bytes."""
+    of SA_t, rounded once to wl.dtype).  Y_k = S_B Z_k is exact and is put on the
+    2^-Y_BITS grid (clipped to |y| <= Y_CLIP) before the second product, which is then
+    exact too.  Samples are drawn per generator chunk of CHUNK_ROWS // 64 samples, so any
+    k0..k1 reproduce the same bytes."""
     per = max(1, CHUNK_ROWS // 64)
     out = []
     dev = SA_t.device
@@ -147,10 +172,12 @@ def matrix_sample_chunk(wl: Workload, seed: int, k0: int, k1: int, SA_t: torch.T
     for c in range(c0, c1 + 1):
         a = c * per
         rows = min(wl.N, a + per) - a
-        z = _rng(seed, _ZK, c).standard_normal((rows, wl.m, wl.n))
+        z = _normals(seed, _ZK, c, (rows, wl.m, wl.n))
         lo, hi = max(k0, a) - a, min(k1, a + rows) - a
         zt = torch.from_numpy(z[lo:hi]).to(dev)
-        out.append(_round_to(torch.matmul(torch.matmul(SB_t, zt), SA_t.t()), wl.torch_dtype))
+        y = torch.matmul(SB_t, zt).clamp_(-Y_CLIP, Y_CLIP)
+        y = torch.round(y * (2.0 ** Y_BITS)) * (2.0 ** -Y_BITS)
+        out.append(_round_to(torch.matmul(y, SA_t.t()), wl.torch_dtype))
     return torch.cat(out, 0)
 
 

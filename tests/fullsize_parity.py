@@ -122,11 +122,14 @@ def oracle_source_digest() -> str:
         return hashlib.sha256(f.read()).hexdigest()
 
 
-def oracle_fit_cached(name: str, wl, X, G, digest: str, cache: str):
+def oracle_fit_cached(name: str, wl, X, G, digest: str, cache: str, tol: float = 0.0):
+    """The oracle fit of the workload (all wl.iters iterations, or until delta_t < tol:
+    past the fixed point further iterations move the factors by less than tol)."""
     import oracle
 
     os.makedirs(cache, exist_ok=True)
-    path = os.path.join(cache, f"{name}_{digest[:16]}_{oracle_source_digest()[:12]}.npz")
+    tag = "" if tol == 0.0 else f"_tol{tol:g}"
+    path = os.path.join(cache, f"{name}_{digest[:16]}_{oracle_source_digest()[:12]}{tag}.npz")
     if os.path.exists(path):
         z = np.load(path)
         return z["A"], z["B"], float(z["seconds"]), json.loads(str(z["deltas"]))
@@ -136,7 +139,7 @@ def oracle_fit_cached(name: str, wl, X, G, digest: str, cache: str):
         print(f"  [{name}] oracle iteration {t}/{wl.iters} done at {time.time() - t0:.0f} s "
               f"(delta {delta:.3e})", flush=True)
 
-    fit = oracle.flipflop_fit(X, G, iters=wl.iters, progress=progress)
+    fit = oracle.flipflop_fit(X, G, iters=wl.iters, tol=tol, progress=progress)
     sec = time.time() - t0
     deltas = [None if math.isinf(d) else d for d in fit.deltas]
     np.savez(path, A=fit.A, B=fit.B, seconds=sec, deltas=json.dumps(deltas))
@@ -192,8 +195,9 @@ def run_oracle(args) -> int:
         X, G = portable.rank_one_samples(wl, seed=SEED, device="cpu")
         digest = portable.sha256(X, G)
         t_gen = time.time() - t0
+        tol = args.oracle_tol if name in args.tol_configs else 0.0
         if args.fit_only:
-            _, _, sec, _ = oracle_fit_cached(name, wl, X, G, digest, args.cache)
+            _, _, sec, _ = oracle_fit_cached(name, wl, X, G, digest, args.cache, tol)
             print(json.dumps({"workload": name, "sha256": digest, "oracle_fit_s": sec,
                               "host_gen_s": t_gen}), flush=True)
             del X, G
@@ -206,11 +210,12 @@ def run_oracle(args) -> int:
                               "gpu": rec["sha256"], "host": digest}), flush=True)
             status = 1
             continue
-        A_ref, B_ref, sec, deltas = oracle_fit_cached(name, wl, X, G, digest, args.cache)
+        A_ref, B_ref, sec, deltas = oracle_fit_cached(name, wl, X, G, digest, args.cache, tol)
         cmp = compare(rec, arr, A_ref, B_ref)
         line = {"workload": name, "N": wl.N, "n": wl.n, "m": wl.m, "iters": wl.iters,
                 "dtype": wl.dtype, "sha256": digest, **cmp,
                 "gpu_fit_ms": rec["fit_ms"], "oracle_fit_s": sec,
+                "oracle_iters": len(deltas), "oracle_last_delta": deltas[-1],
                 "oracle_cores": len(os.sched_getaffinity(0)), "host_gen_s": t_gen,
                 "tolerance": 2e-3, "pass": cmp["kron_rel_err_2se_upper"] <= 2e-3}
         print(json.dumps(line), flush=True)
@@ -227,10 +232,16 @@ def main() -> int:
     p.add_argument("--out", default=os.path.join(ROOT, "gpurun_out", "parity"))
     p.add_argument("--gpu", default=os.path.join(ROOT, "gpurun_out", "parity"))
     p.add_argument("--cache", default=os.path.join(ROOT, "tests", ".oracle_cache"))
+    p.add_argument("--oracle-tol", type=float, default=1e-12,
+                   help="oracle stopping tolerance for the --tol-configs workloads")
+    p.add_argument("--tol-configs", default="llama3_8b_down_14336x4096",
+                   help="workloads whose oracle fit stops at --oracle-tol (the rest run "
+                        "all their iterations)")
     p.add_argument("--fit-only", action="store_true",
                    help="oracle half: only run (and cache) the oracle fits")
     args = p.parse_args()
     args.configs = [c for c in args.configs.split(",") if c]
+    args.tol_configs = [c for c in args.tol_configs.split(",") if c]
     for c in args.configs:
         if synth.WORKLOADS[c].kind != "rank_one":
             raise SystemExit(f"{c}: only rank-one workloads are compared by this script")
