@@ -329,6 +329,53 @@ def flipflop_fit_matrix(Gk, iters: int, tol: float = 0.0, damping: float = 0.0,
     return FitResult(A=A, B=B, iters_done=t_done, deltas=deltas, loglik=lls, mean_qr=mqr)
 
 
+def flipflop_fit_matrix_blocks(sample_blocks, N: int, m: int, n: int, iters: int,
+                               tol: float = 0.0, damping: float = 0.0, progress=None):
+    """flipflop_fit_matrix for samples too large to hold at once: sample_blocks() yields
+    consecutive blocks G_k (b x m x n, any float dtype) covering all N samples, and may
+    be called once per half-step.  Same updates, constants, order and normalisation; each
+    expectation is accumulated block by block.  Returns (A, B, iters_done, deltas); the
+    log-likelihood statistics are not evaluated."""
+    A = np.eye(n)
+    B_prev, A_prev = None, A.copy()
+    deltas = []
+    t_done = 0
+    B = None
+    for t in range(1, iters + 1):
+        LA = cholesky(A)
+        # B = 1/(N n) sum_k G_k A^-1 G_k^T = sum_k W_k^T W_k with W_k = L_A^-1 G_k^T
+        acc = np.zeros((m, m))
+        for Gb in sample_blocks():
+            Gb = as_f64(Gb)
+            b = Gb.shape[0]
+            W = sla.solve_triangular(LA, Gb.transpose(2, 0, 1).reshape(n, b * m), lower=True)
+            W = W.reshape(n, b, m).transpose(1, 0, 2).reshape(b * n, m)   # rows (k, i)
+            acc += W.T @ W
+        B = damp(acc / (N * n), damping)
+        LB = cholesky(B)
+        # A = 1/(N m) sum_k G_k^T B^-1 G_k = sum_k Y_k^T Y_k with Y_k = L_B^-1 G_k
+        acc = np.zeros((n, n))
+        for Gb in sample_blocks():
+            Gb = as_f64(Gb)
+            b = Gb.shape[0]
+            Y = sla.solve_triangular(LB, Gb.transpose(1, 0, 2).reshape(m, b * n), lower=True)
+            Y = Y.reshape(m, b, n).transpose(1, 0, 2).reshape(b * m, n)   # rows (k, j)
+            acc += Y.T @ Y
+        A = damp(acc / (N * m), damping)
+        s = np.trace(A) / n
+        A, B = A / s, B * s
+        delta = math.inf if B_prev is None else max(rel_change(A, A_prev),
+                                                    rel_change(B, B_prev))
+        deltas.append(delta)
+        A_prev, B_prev = A.copy(), B.copy()
+        t_done = t
+        if progress is not None:
+            progress(t, delta)
+        if tol > 0.0 and delta < tol:
+            break
+    return A, B, t_done, deltas
+
+
 def _sum_sq_two_sided(Y: np.ndarray, LA: np.ndarray) -> float:
     """sum_k ||Y_k L_A^-T||_F^2 for Y of shape (m, N, n)."""
     m, N, n = Y.shape

@@ -181,6 +181,44 @@ def matrix_sample_chunk(wl: Workload, seed: int, k0: int, k1: int, SA_t: torch.T
     return torch.cat(out, 0)
 
 
+def matrix_blocks(wl: Workload, seed: int = 0, device="cpu", N: Optional[int] = None):
+    """Yield (k0, block) over all samples of the matrix workload in generator chunks of
+    CHUNK_ROWS // 64 samples (G_k = S_B Z_k S_A^T exactly as matrix_sample_chunk), the
+    normals of the next chunks drawn by a thread pool meanwhile."""
+    assert wl.kind == "matrix"
+    N = wl.N if N is None else int(N)
+    dev = torch.device(device)
+    SA, SB = matrix_normal_factors(wl, seed)
+    SA_t, SB_t = torch.from_numpy(SA).to(dev), torch.from_numpy(SB).to(dev)
+    per = max(1, CHUNK_ROWS // 64)
+    nchunks = (N + per - 1) // per
+
+    def draw(c):
+        rows = min(N, (c + 1) * per) - c * per
+        return _normals(seed, _ZK, c, (rows, wl.m, wl.n))
+
+    with ThreadPoolExecutor(_threads()) as ex:
+        ahead = max(2, _threads())
+        futs = [ex.submit(draw, c) for c in range(min(nchunks, ahead))]
+        for c in range(nchunks):
+            z = futs[c].result()
+            futs[c] = None
+            if c + ahead < nchunks:
+                futs.append(ex.submit(draw, c + ahead))
+            y = torch.matmul(SB_t, torch.from_numpy(z).to(dev)).clamp_(-Y_CLIP, Y_CLIP)
+            y = torch.round(y * (2.0 ** Y_BITS)) * (2.0 ** -Y_BITS)
+            yield c * per, _round_to(torch.matmul(y, SA_t.t()), wl.torch_dtype)
+
+
+def matrix_samples(wl: Workload, seed: int = 0, device="cpu", N: Optional[int] = None):
+    """All N matrix samples (N x m x n, dtype wl.dtype) on `device`, drawn portably."""
+    N = wl.N if N is None else int(N)
+    out = torch.empty(N, wl.m, wl.n, dtype=wl.torch_dtype, device=device)
+    for k0, blk in matrix_blocks(wl, seed, device, N):
+        out[k0:k0 + blk.shape[0]] = blk
+    return out
+
+
 def sha256(*tensors: torch.Tensor, chunk_bytes: int = 1 << 28) -> str:
     """Digest of the raw bytes of the tensors, in order (row-major, as stored)."""
     h = hashlib.sha256()

@@ -44,8 +44,8 @@ import torch  # noqa: E402
 import synth  # noqa: E402
 from synth import portable  # noqa: E402
 
-RANK_ONE = ["tiny_64", "llama7b_attn_4096", "llama7b_mlp_up_4096x11008",
-            "llama3_8b_down_14336x4096"]
+ALL = ["tiny_64", "kron_recovery_512x768", "llama7b_attn_4096", "llama7b_mlp_up_4096x11008",
+       "llama3_8b_down_14336x4096"]
 SKETCH_K = 64
 FULL_MAX_D = 1024      # factors up to this size are saved whole
 SEED = 0
@@ -77,16 +77,28 @@ def run_gpu(args) -> int:
     for name in args.configs:
         wl = synth.WORKLOADS[name]
         t0 = time.time()
-        X, G = portable.rank_one_samples(wl, seed=SEED, device="cuda")
+        matrix = wl.kind == "matrix"
+        if matrix:
+            Gk = portable.matrix_samples(wl, seed=SEED, device="cuda")
+            data = (Gk,)
+        else:
+            X, G = portable.rank_one_samples(wl, seed=SEED, device="cuda")
+            data = (X, G)
         torch.cuda.synchronize()
         t_gen = time.time() - t0
-        digest = portable.sha256(X, G)
+        digest = portable.sha256(*data)
+
+        def fit(h):
+            if matrix:
+                return h.fit_matrix(Gk, wl.iters)
+            return h.fit(X, G, iters=wl.iters)
+
         with ffh.Handle(dtype=wl.dtype) as h:
-            A, B = h.fit(X, G, iters=wl.iters)
+            A, B = fit(h)
             torch.cuda.synchronize()
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record()
-            A, B = h.fit(X, G, iters=wl.iters)
+            A, B = fit(h)
             e1.record()
             torch.cuda.synchronize()
             stats = h.stats()
@@ -109,7 +121,8 @@ def run_gpu(args) -> int:
             json.dump(rec, f)
         print(json.dumps({k: v for k, v in rec.items() if k not in ("loglik", "mean_qr")}),
               flush=True)
-        del X, G, A, B
+        del data, A, B
+        X = G = Gk = None
         torch.cuda.empty_cache()
     return 0
 
@@ -122,7 +135,8 @@ def oracle_source_digest() -> str:
         return hashlib.sha256(f.read()).hexdigest()
 
 
-def oracle_fit_cached(name: str, wl, X, G, digest: str, cache: str, tol: float = 0.0):
+def oracle_fit_cached(name: str, wl, X, G, digest: str, cache: str, tol: float = 0.0,
+                      blocks=None):
     """The oracle fit of the workload (all wl.iters iterations, or until delta_t < tol:
     past the fixed point further iterations move the factors by less than tol)."""
     import oracle
@@ -139,11 +153,16 @@ def oracle_fit_cached(name: str, wl, X, G, digest: str, cache: str, tol: float =
         print(f"  [{name}] oracle iteration {t}/{wl.iters} done at {time.time() - t0:.0f} s "
               f"(delta {delta:.3e})", flush=True)
 
-    fit = oracle.flipflop_fit(X, G, iters=wl.iters, tol=tol, progress=progress)
+    if blocks is not None:
+        A, B, _, dl = oracle.flipflop_fit_matrix_blocks(blocks, wl.N, wl.m, wl.n, wl.iters,
+                                                        tol=tol, progress=progress)
+    else:
+        fit = oracle.flipflop_fit(X, G, iters=wl.iters, tol=tol, progress=progress)
+        A, B, dl = fit.A, fit.B, fit.deltas
     sec = time.time() - t0
-    deltas = [None if math.isinf(d) else d for d in fit.deltas]
-    np.savez(path, A=fit.A, B=fit.B, seconds=sec, deltas=json.dumps(deltas))
-    return fit.A, fit.B, sec, deltas
+    deltas = [None if math.isinf(d) else d for d in dl]
+    np.savez(path, A=A, B=B, seconds=sec, deltas=json.dumps(deltas))
+    return A, B, sec, deltas
 
 
 def sketch_err2(sketch_gpu: np.ndarray, F_ref: np.ndarray):
@@ -192,12 +211,26 @@ def run_oracle(args) -> int:
     for name in args.configs:
         wl = synth.WORKLOADS[name]
         t0 = time.time()
-        X, G = portable.rank_one_samples(wl, seed=SEED, device="cpu")
-        digest = portable.sha256(X, G)
+        blocks = None
+        if wl.kind == "matrix":
+            # 103 GB of samples at the full size: drawn block by block on every pass
+            X = G = None
+
+            def blocks(wl=wl):
+                for _, blk in portable.matrix_blocks(wl, seed=SEED, device="cpu"):
+                    yield blk
+
+            hsh = hashlib.sha256()
+            for blk in blocks():
+                hsh.update(blk.contiguous().view(-1).view(torch.uint8).numpy().tobytes())
+            digest = hsh.hexdigest()
+        else:
+            X, G = portable.rank_one_samples(wl, seed=SEED, device="cpu")
+            digest = portable.sha256(X, G)
         t_gen = time.time() - t0
         tol = args.oracle_tol if name in args.tol_configs else 0.0
         if args.fit_only:
-            _, _, sec, _ = oracle_fit_cached(name, wl, X, G, digest, args.cache, tol)
+            _, _, sec, _ = oracle_fit_cached(name, wl, X, G, digest, args.cache, tol, blocks)
             print(json.dumps({"workload": name, "sha256": digest, "oracle_fit_s": sec,
                               "host_gen_s": t_gen}), flush=True)
             del X, G
@@ -210,7 +243,8 @@ def run_oracle(args) -> int:
                               "gpu": rec["sha256"], "host": digest}), flush=True)
             status = 1
             continue
-        A_ref, B_ref, sec, deltas = oracle_fit_cached(name, wl, X, G, digest, args.cache, tol)
+        A_ref, B_ref, sec, deltas = oracle_fit_cached(name, wl, X, G, digest, args.cache, tol,
+                                                      blocks)
         cmp = compare(rec, arr, A_ref, B_ref)
         line = {"workload": name, "N": wl.N, "n": wl.n, "m": wl.m, "iters": wl.iters,
                 "dtype": wl.dtype, "sha256": digest, **cmp,
@@ -228,13 +262,13 @@ def run_oracle(args) -> int:
 def main() -> int:
     p = argparse.ArgumentParser()
     p.add_argument("half", choices=["gpu", "oracle"])
-    p.add_argument("--configs", default=",".join(RANK_ONE))
+    p.add_argument("--configs", default=",".join(ALL))
     p.add_argument("--out", default=os.path.join(ROOT, "gpurun_out", "parity"))
     p.add_argument("--gpu", default=os.path.join(ROOT, "gpurun_out", "parity"))
     p.add_argument("--cache", default=os.path.join(ROOT, "tests", ".oracle_cache"))
     p.add_argument("--oracle-tol", type=float, default=1e-12,
                    help="oracle stopping tolerance for the --tol-configs workloads")
-    p.add_argument("--tol-configs", default="llama3_8b_down_14336x4096",
+    p.add_argument("--tol-configs", default="llama3_8b_down_14336x4096,kron_recovery_512x768",
                    help="workloads whose oracle fit stops at --oracle-tol (the rest run "
                         "all their iterations)")
     p.add_argument("--fit-only", action="store_true",
@@ -242,9 +276,6 @@ def main() -> int:
     args = p.parse_args()
     args.configs = [c for c in args.configs.split(",") if c]
     args.tol_configs = [c for c in args.tol_configs.split(",") if c]
-    for c in args.configs:
-        if synth.WORKLOADS[c].kind != "rank_one":
-            raise SystemExit(f"{c}: only rank-one workloads are compared by this script")
     return run_gpu(args) if args.half == "gpu" else run_oracle(args)
 
 

@@ -344,6 +344,25 @@ def test_row_blocks_do_not_change_the_fit():
     assert rel(fb.A, fr.A) < 1e-12 and rel(fb.B, fr.B) < 1e-12
 
 
+def test_matrix_fit_over_sample_blocks_equals_matrix_fit():
+    """The block-accumulated matrix fit (samples drawn block by block) is the same fit:
+    sums over samples grouped differently, including a ragged last block."""
+    N, m, n = 37, 5, 4
+    rng = np.random.default_rng(31)
+    Gk = rng.standard_normal((N, m, n)) * (1.0 + np.abs(rng.standard_normal((N, 1, 1))))
+    ref = oracle.flipflop_fit_matrix(Gk, iters=6, damping=0.05)
+
+    def blocks():
+        for k0 in range(0, N, 10):
+            yield Gk[k0:k0 + 10]
+
+    A, B, t, deltas = oracle.flipflop_fit_matrix_blocks(blocks, N, m, n, iters=6, damping=0.05)
+    assert t == 6
+    assert np.linalg.norm(A - ref.A) / np.linalg.norm(ref.A) < 1e-12
+    assert np.linalg.norm(B - ref.B) / np.linalg.norm(ref.B) < 1e-12
+    assert np.allclose(deltas[1:], ref.deltas[1:], rtol=1e-8)
+
+
 def test_tol_stops_early():
     N, n, m = 300, 4, 3
     X = _correlated(N, n, seed=13, stream=0)
