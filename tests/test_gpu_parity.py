@@ -60,6 +60,29 @@ def test_weighted_gram_matches_oracle(N, d, weighted):
     assert np.all(np.abs(Cn - ref) <= bound), np.max(np.abs(Cn - ref) / bound)
 
 
+@pytest.mark.parametrize("N,d", [(2048, 4096), (4097, 4096), (9000, 4096), (5000, 4000)])
+def test_streamed_weighted_gram_matches_oracle(N, d):
+    """Widths whose 256 x 256 lower-triangle tiles about fill the GPU (d about 4096) take the
+    streamed kernel: one CTA per tile, the weighted operand written a chunk of 2048 samples
+    ahead into a 3-slot ring (N = 9000 reuses the slots, 4097 and 5000 end in a partial
+    chunk, d = 4000 in a partial tile).  Same elementwise bound as the split-K kernel."""
+    wl = synth.WORKLOADS["llama7b_attn_4096"].with_(n=d, m=8)
+    X, _ = synth.rank_one_samples(wl, seed=7, device="cuda", N=N)
+    w = torch.rand(N, device="cuda", generator=torch.Generator("cuda").manual_seed(8)) * 3
+    scale = 1.0 / (N * 5)
+    with ffh.Handle(dtype="bf16") as h:
+        C = h.weighted_gram(X, w, scale)
+        C2 = h.weighted_gram(X, w, scale)
+    torch.cuda.synchronize()
+    assert torch.equal(C, C2), "the streamed Gram must be deterministic"
+    Vn, wn = oracle.as_f64(X), oracle.as_f64(w)
+    ref = oracle.weighted_gram(Vn, wn, scale)
+    Cn = oracle.as_f64(C)
+    assert np.array_equal(Cn, Cn.T), "output must be exactly symmetric"
+    bound = _bf16_gram_bound(Vn, wn, scale) + 1e-7 * np.abs(ref).max()
+    assert np.all(np.abs(Cn - ref) <= bound), np.max(np.abs(Cn - ref) / bound)
+
+
 def test_weighted_gram_f32_input():
     N, d = 2000, 100          # fp32 input: any d (internally padded to a multiple of 8)
     X = synth.gaussian(N, d, seed=3, device="cuda")
