@@ -75,7 +75,7 @@ def measured_peaks():
 
 def gram_source_sha256() -> str:
     """sha256 of the Gram kernel's source: kernels_tc.cu from `namespace gram {` up to the
-    quadratic-form section (kernel, tile tables, reduction, launch)."""
+    quadratic-form section (kernel, tile tables, reduction, launcher)."""
     src = os.path.join(ROOT, "paper_2609_14706_gb300", "csrc", "kernels_tc.cu")
     with open(src) as f:
         text = f.read()
@@ -84,10 +84,10 @@ def gram_source_sha256() -> str:
     return hashlib.sha256(text[a:b].encode()).hexdigest()
 
 
-def profiled_traffic(workload: str):
+def profiled_traffic(workload: str, kernel: str = "k_gram_tc"):
     """DRAM bytes per launch of the Gram kernel from the committed ncu summary, if the
     kernel source is still the one that was profiled (else None)."""
-    path = os.path.join(ROOT, "profiles", f"k_gram_tc_{workload}.md")
+    path = os.path.join(ROOT, "profiles", f"{kernel}_{workload}.md")
     try:
         text = open(path).read()
     except OSError:
@@ -363,9 +363,10 @@ def run_ours(args):
     qform_tflops = ((qform_flops_step * args.steps) / (tim["qform_ms"] / 1e3) / 1e12
                     if tim["qform_ms"] > 0 else None)
     roofline = {"bound": "tensor",
-                "kernel": "k_gram_tc (weighted Gram, diag(w) applied in its operand load)",
+                "kernel": "k_gram_tc (weighted Gram, diag(w) applied inside the kernel)",
                 "achieved": gram_tflops, "peak": peak, "unit": "TFLOP/s",
-                "frac": gram_tflops / peak, "traffic": profiled_traffic(wl.name),
+                "frac": gram_tflops / peak,
+                "traffic": profiled_traffic(wl.name),
                 "traffic_unit": "bytes per launch (ncu dram__bytes_read + write)",
                 "peak_source": f"{peak_kind} bf16 dense, sustained (kernel timed inside a long step)",
                 "flops_per_launch": gram_flops_step * args.steps / max(1, tim["gram_launches"]),

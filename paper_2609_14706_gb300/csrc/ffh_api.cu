@@ -19,7 +19,6 @@
 #include <cstddef>
 #include <cstdio>
 #include <cstring>
-#include <initializer_list>
 #include <string>
 #include <vector>
 
@@ -298,31 +297,15 @@ ffh_status stage_input(ffh_t h, const void* V, bool on_dev, int64_t N, int64_t d
 }
 
 // C = scale * V^T diag(w) V on the tensor cores; the weights enter the kernel's operand
-// load (no scaled copy of V).  With a ring (gram_stream_ring_bytes) and a d whose tiles
-// about fill the GPU, the streamed kernel (one CTA per tile, no split-K reduction) runs.
+// load (no scaled copy of V).
 ffh_status gram(ffh_t h, const Staged& V, int64_t N, int64_t d, const float* w_padded, float scale,
-                float* C, float* partial, const GramTables& gt, DevStatus* st,
-                void* ring = nullptr) {
+                float* C, float* partial, const GramTables& gt, DevStatus* st) {
   cudaEvent_t t0 = prof_begin(h);
   cudaEvent_t t1 = t0 ? next_event(h) : nullptr;
-  if (ring && w_padded && h->opt.fault == FFH_FAULT_NONE && gram_stream_eligible(d, num_sms())) {
-    CK(launch_gram_stream(V.bf, N, d, V.ld_bf, w_padded, scale, C, d, ring, gt.tiles, gt.plan.T,
-                          st, h->stream));
-    prof_end(h, PROF_GRAM, t0);
-    return FFH_OK;
-  }
   CK(launch_gram_tc(V.bf, N, d, V.ld_bf, w_padded, scale, C, d, partial, gt.tiles, gt.lut,
                     gt.plan, st, h->opt.fault, h->stream, t1));
   prof_end(h, PROF_GRAM, t0, t1);
   return FFH_OK;
-}
-
-// ring bytes for the streamed weighted Gram of any of the widths (0 if none is eligible)
-size_t stream_ring_bytes(std::initializer_list<int64_t> widths) {
-  size_t b = 0;
-  for (int64_t d : widths)
-    if (gram_stream_eligible(d, num_sms())) b = std::max(b, gram_stream_ring_bytes(d));
-  return b;
 }
 
 // q_k = ||L^T v_k||^2 = v_k^T F v_k for F = L L^T (the Frobenius variant's weights)
@@ -408,7 +391,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
                     __nv_bfloat16** Gb, float** stage, float** q, float** r, float** A2,
                     float** B2, float** L, float** Linv, __nv_bfloat16** Mb, float** work,
                     int2** tn, int** ln, int2** tm, int** lm, float** partial,
-                    double** trb, float** Ares, float** Bres, void** ring) {
+                    double** trb, float** Ares, float** Bres) {
     *st = c.take<DevStatus>(1);
     *recs = c.take<IterRecord>(iters + 2);
     const bool xcopy = dtype == FFH_F32 || (dtype == FFH_BF16 && !x_dev);
@@ -433,12 +416,9 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
     *trb = c.take<double>(8 + kRedDoubles);  // statistics, then the reduction scratch
     *Ares = c.take<float>((size_t)n * n);
     *Bres = c.take<float>((size_t)m * m);
-    const size_t rb = stream_ring_bytes({n, m});
-    *ring = rb ? c.take<char>(rb) : nullptr;
   };
   DevStatus* st;
   IterRecord* recs;
-  void* ring;
   __nv_bfloat16 *Xb, *Gb, *Mb;
   float *stage, *q, *r, *A2, *B2, *L, *Linv, *work, *partial, *Ares, *Bres;
   int2 *tn, *tm;
@@ -447,13 +427,13 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
   {
     Carve c(nullptr);
     layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &tn,
-           &ln, &tm, &lm, &partial, &trb, &Ares, &Bres, &ring);
+           &ln, &tm, &lm, &partial, &trb, &Ares, &Bres);
     ffh_status es = ensure_ws(h, c.off + 1024);
     if (es) return es;
   }
   Carve c(h->ws);
   layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &tn, &ln,
-         &tm, &lm, &partial, &trb, &Ares, &Bres, &ring);
+         &tm, &lm, &partial, &trb, &Ares, &Bres);
   cudaStream_t s = h->stream;
   // the small kernels of this fit test its status block (see launch_iter_end)
   GateScope gate(st);
@@ -529,7 +509,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
       if (t > 1) CK(launch_dot(q, r, N, &recs[t - 1].sum_qr_A, trb + 8, s));
     }
     // ---- B-update
-    es = gram(h, gs, N, m, q, sB, B[nxt], partial, gtm, st, ring);
+    es = gram(h, gs, N, m, q, sB, B[nxt], partial, gtm, st);
     if (es) return es;
     if (frob) {
       CK(launch_frob2(A[cur], n, trb + 4, trb + 8, s));
@@ -548,7 +528,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
     if (es) return es;
     CK(launch_dot(q, r, N, &R->sum_qr_B, trb + 8, s));
     // ---- A-update
-    es = gram(h, xs, N, n, r, sA, A[nxt], partial, gtn, st, ring);
+    es = gram(h, xs, N, n, r, sA, A[nxt], partial, gtn, st);
     if (es) return es;
     if (frob) {
       CK(launch_frob2(B[nxt], m, trb + 5, trb + 8, s));
@@ -871,10 +851,8 @@ extern "C" ffh_status ffh_weighted_gram(ffh_t h, const void* V, const float* w, 
   const int64_t Npad = (N + 63) / 64 * 64 + 64;
   GramPlan plan = gram_plan(N, d, num_sms());
   auto layout = [&](Carve& c, DevStatus** st, float** wp, __nv_bfloat16** Vb, float** partial,
-                    int2** tiles, int** lut, void** ring) {
+                    int2** tiles, int** lut) {
     *st = c.take<DevStatus>(1);
-    const size_t rb = w ? stream_ring_bytes({d}) : 0;
-    *ring = rb ? c.take<char>(rb) : nullptr;
     *wp = c.take<float>(Npad);
     *Vb = (dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(d)) : nullptr;
     *partial = c.take<float>(gram_partial_bytes(plan) / 4);
@@ -886,15 +864,14 @@ extern "C" ffh_status ffh_weighted_gram(ffh_t h, const void* V, const float* w, 
   __nv_bfloat16* Vb;
   int2* tiles;
   int* lut;
-  void* ring;
   {
     Carve c(nullptr);
-    layout(c, &st, &wp, &Vb, &partial, &tiles, &lut, &ring);
+    layout(c, &st, &wp, &Vb, &partial, &tiles, &lut);
     ffh_status es = ensure_ws(h, c.off + 1024);
     if (es) return es;
   }
   Carve c(h->ws);
-  layout(c, &st, &wp, &Vb, &partial, &tiles, &lut, &ring);
+  layout(c, &st, &wp, &Vb, &partial, &tiles, &lut);
   cudaStream_t s = h->stream;
   CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
   const float* wuse = nullptr;
@@ -909,7 +886,7 @@ extern "C" ffh_status ffh_weighted_gram(ffh_t h, const void* V, const float* w, 
   GramTables gt;
   es = setup_tables(h, N, d, &gt, tiles, lut);
   if (es) return es;
-  es = gram(h, vs_, N, d, wuse, scale, C_out, partial, gt, st, ring);
+  es = gram(h, vs_, N, d, wuse, scale, C_out, partial, gt, st);
   if (es) return es;
   return read_status(h, st);
 }
@@ -1190,10 +1167,8 @@ extern "C" ffh_status ffh_partial_gram(ffh_t h, const void* U, const void* V, in
   GramPlan plan = gram_plan(N, dv, num_sms());
   auto layout = [&](Carve& c, DevStatus** st, __nv_bfloat16** Ub, __nv_bfloat16** Vb, float** w,
                     float** L, float** Linv, __nv_bfloat16** Mb, float** work, float** partial,
-                    int2** tiles, int** lut, float** Ptmp, void** ring) {
+                    int2** tiles, int** lut, float** Ptmp) {
     *st = c.take<DevStatus>(1);
-    const size_t rb = stream_ring_bytes({dv});
-    *ring = rb ? c.take<char>(rb) : nullptr;
     *Ub = (dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(du)) : nullptr;
     *Vb = (dtype == FFH_F32) ? c.take<__nv_bfloat16>((size_t)N * pad8(dv)) : nullptr;
     *w = c.take<float>(Npad);
@@ -1211,15 +1186,14 @@ extern "C" ffh_status ffh_partial_gram(ffh_t h, const void* U, const void* V, in
   float *w, *L, *Linv, *work, *partial, *Ptmp;
   int2* tiles;
   int* lut;
-  void* ring;
   {
     Carve c(nullptr);
-    layout(c, &st, &Ub, &Vb, &w, &L, &Linv, &Mb, &work, &partial, &tiles, &lut, &Ptmp, &ring);
+    layout(c, &st, &Ub, &Vb, &w, &L, &Linv, &Mb, &work, &partial, &tiles, &lut, &Ptmp);
     ffh_status es = ensure_ws(h, c.off + 1024);
     if (es) return es;
   }
   Carve c(h->ws);
-  layout(c, &st, &Ub, &Vb, &w, &L, &Linv, &Mb, &work, &partial, &tiles, &lut, &Ptmp, &ring);
+  layout(c, &st, &Ub, &Vb, &w, &L, &Linv, &Mb, &work, &partial, &tiles, &lut, &Ptmp);
   cudaStream_t s = h->stream;
   CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
   CK(cudaMemsetAsync(w, 0, sizeof(float) * Npad, s));
@@ -1240,7 +1214,7 @@ extern "C" ffh_status ffh_partial_gram(ffh_t h, const void* U, const void* V, in
   GramTables gt;
   es = setup_tables(h, N, dv, &gt, tiles, lut);
   if (es) return es;
-  es = gram(h, vs_, N, dv, w, 1.0f, accumulate ? Ptmp : P_out, partial, gt, st, ring);
+  es = gram(h, vs_, N, dv, w, 1.0f, accumulate ? Ptmp : P_out, partial, gt, st);
   if (es) return es;
   if (accumulate) CK(launch_add(P_out, Ptmp, dv * dv, s));
   DevStatus hst;

@@ -178,16 +178,6 @@ cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t
                            float* partial, int2* tiles_dev, int* tile_lut_dev,
                            const GramPlan& plan, DevStatus* st, int fault, cudaStream_t s,
                            cudaEvent_t after_main = nullptr);
-// Streamed weighted Gram (one CTA per lower-triangle tile, weights applied to a ring of
-// sample chunks in L2 by the CTAs themselves, no split-K reduction): eligible when the
-// tiles about fill the GPU; `ring` holds gram_stream_ring_bytes(d) bytes (256-aligned);
-// `tiles_dev` is the tile table of gram_build_tiles (T entries).  C = scale V^T diag(w) V,
-// full symmetric.
-bool gram_stream_eligible(int64_t d, int sms);
-size_t gram_stream_ring_bytes(int64_t d);
-cudaError_t launch_gram_stream(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t ld,
-                               const float* w, float scale, float* C, int64_t ldc, void* ring,
-                               const int2* tiles_dev, int T, DevStatus* st, cudaStream_t s);
 // q_k = ||M v_k||^2, V bf16 N x d (pitch ld), M bf16 d x d lower (pitch ldm)
 cudaError_t launch_qform_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t ld,
                             const __nv_bfloat16* M, int64_t ldm, float* q, DevStatus* st,

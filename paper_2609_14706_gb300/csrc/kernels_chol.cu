@@ -1233,6 +1233,60 @@ void chol_streams_destroy(CholStreams* cs) {
   if (cs->side) cudaStreamDestroy(cs->side), cs->side = nullptr;
 }
 
+// M = L^-1 by recursive doubling over block size b = 128, 256, ... (the 128 x 128 diagonal
+// blocks of M already hold the leaf kernels' inverses); T and the split buffers are scratch.
+// From this order on the look-ahead schedule pairs the panels of the trailing update
+// (the fp32 trailing matrix no longer fits in L2, so its traffic bounds the factorization)
+constexpr int64_t kGroupedMinD = 8192;
+
+static cudaError_t cholesky_inverse(const float* L, float* Linv, int64_t d, float* T,
+                                    __nv_bfloat16* const* sb, DevStatus* st, cudaStream_t s) {
+  cudaError_t e;
+  if (!Linv) return cudaSuccess;
+  for (int64_t b = LB; b < d; b *= 2) {
+    const int64_t full_pairs = d / (2 * b);
+    const int64_t o_last = full_pairs * 2 * b;
+    const int64_t rows_last = d - o_last - b;
+    for (int part = 0; part < 2; ++part) {
+      const int batch = (int)(part == 0 ? full_pairs : (rows_last > 0 ? 1 : 0));
+      if (batch == 0) continue;
+      const int64_t o = part == 0 ? 0 : o_last;
+      const int rows = (int)(part == 0 ? b : rows_last);
+      const int64_t zs = 2 * b * d + 2 * b;  // source stride between pairs
+      const int kb = (int)((b + 63) / 64 * 64);
+      const int kr = (rows + 63) / 64 * 64;
+      const int rp = (rows + 127) / 128 * 128;
+      const int bp = (int)((b + 127) / 128 * 128);
+      // T_z = L21_z M11_z : A' = split(L21) (rows x b), B' = split(M11^T) (b x b)
+      Split l21{sb[0], rp, kb, batch};
+      Split m11t{sb[1], bp, kb, batch};
+      if ((e = split(L + (o + b) * d + o, d, zs, rows, (int)b, false, l21, s)) != cudaSuccess)
+        return e;
+      if ((e = split(Linv + o * d + o, d, zs, (int)b, (int)b, true, m11t, s)) != cudaSuccess)
+        return e;
+      const int as1[3] = {0, 0, kb}, bs1[3] = {0, kb, 0};
+      // B' = M11^T is upper triangular: output column block c needs k >= c
+      if ((e = gemm_tc(l21, m11t, 3, as1, bs1, (int)b, T, b, (int64_t)rp * b, rows, (int)b, 1.f,
+                       0.f, false, batch, st, s, nullptr, TRI_K_FROM_COL)) != cudaSuccess)
+        return e;
+      // M21_z = -M22_z T_z : A' = split(M22) (rows x rows), B' = split(T^T) (b x rows)
+      Split m22{sb[2], rp, kr, batch};
+      Split tt{sb[3], bp, kr, batch};
+      if ((e = split(Linv + (o + b) * d + (o + b), d, zs, rows, rows, false, m22, s)) !=
+          cudaSuccess)
+        return e;
+      // B'[c][k] = T[k][c]: b output rows, `rows` output columns
+      if ((e = split(T, b, (int64_t)rp * b, (int)b, rows, true, tt, s)) != cudaSuccess) return e;
+      const int as2[3] = {0, 0, kr}, bs2[3] = {0, kr, 0};
+      // A' = M22 is lower triangular: output row block r needs k < r + 128
+      if ((e = gemm_tc(m22, tt, 3, as2, bs2, rows, Linv + (o + b) * d + o, d, zs, rows, (int)b,
+                       -1.f, 0.f, false, batch, st, s, nullptr, TRI_K_TO_ROW)) != cudaSuccess)
+        return e;
+    }
+  }
+  return cudaSuccess;
+}
+
 static cudaError_t cholesky_tc_body(const float* F, int64_t d, int64_t ldf, float* L, float* Linv,
                                     void* work, DevStatus* st, int fault, cudaStream_t s,
                                     CholStreams* cs);
@@ -1297,6 +1351,83 @@ static cudaError_t cholesky_tc_body(const float* F, int64_t d, int64_t ldf, floa
   if ((e = cudaMemsetAsync(&st->logdet, 0, sizeof(double), s)) != cudaSuccess) return e;
   float* Mdiag = Linv ? Linv : T;  // the diagonal-block inverses (T is free until the inverse)
   const int np = (int)((d + LB - 1) / LB);
+  const int aseg[3] = {0, 0, 128}, bseg[3] = {0, 128, 0};
+  if (cs && d >= kGroupedMinD) {
+    // Panels in pairs: the trailing update beyond the next two column blocks applies both
+    // panels at once (K = 256), which halves the passes over the fp32 trailing matrix
+    // (the bound at large d) and the waits on the side stream.  The pair's L21 splits share
+    // one buffer laid out [hi(256) | lo(256)] per row, rows from the first panel's
+    // trailing rows: the first panel's split at K offset 0, the second's at K offset 128
+    // and 128 rows down.
+    const int gseg[3] = {0, 0, 256}, hseg[3] = {0, 256, 0};
+    const int rows_pad_all = (int)((d + 127) / 128 * 128);
+    const int64_t pitch = 512;
+    for (int p = 0; p < np; ++p) {
+      const int64_t o = (int64_t)p * LB;
+      if ((e = launch_pdl(k_chol_leaf, dim3(1), dim3(LEAF_THREADS), LB_SMEM, s, W, d, d, o, L, d,
+                          Mdiag, d, sb[1], st, fault)) != cudaSuccess)
+        return e;
+      note_launches(1);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+      const int rows = (int)(d - o - LB);
+      if (rows <= 0) continue;
+      const bool second = (p & 1) != 0;
+      __nv_bfloat16* pair = sb[2 + 2 * ((p >> 1) & 1)];
+      // solve: L21 = A21 M11^T, its split into the pair buffer
+      Split a21{sb[0] + (size_t)LB * 2 * 128, (int)((rows + 127) / 128 * 128), 128, 1};
+      Split m11{sb[1], 128, 128, 1};
+      if (p == 0 && (e = split(W + (o + LB) * d + o, d, 0, rows, LB, false, a21, s)) != cudaSuccess)
+        return e;
+      Split l21{second ? pair + LB * pitch + 128 : pair, rows_pad_all, 256, 1};
+      if ((e = gemm_tc(a21, m11, 3, aseg, bseg, 128, L + (o + LB) * d + o, d, 0, rows, LB, 1.f,
+                       0.f, false, 1, st, s, &l21)) != cudaSuccess)
+        return e;
+      const int rows_pad = (rows + 127) / 128 * 128;
+      Split next_a21{sb[0], rows_pad + LB, 128, 1};
+      if (!second) {
+        // the next column block with this panel alone (K = 128), after the previous pair's
+        // side update of the columns beyond it
+        if (p > 0 && (e = cudaStreamWaitEvent(s, cs->ev[2 + (((p >> 1) - 1) & 1)], 0)) !=
+                         cudaSuccess)
+          return e;
+        Split v{pair, rows_pad_all, 256, 1};
+        Split head{pair, LB, 256, 1};
+        if ((e = gemm_tc(v, head, 3, gseg, hseg, 128, W + (o + LB) * d + (o + LB), d, 0, rows,
+                         rows < LB ? rows : LB, -1.f, 1.f, true, 1, st, s,
+                         rows > LB ? &next_a21 : nullptr)) != cudaSuccess)
+          return e;
+        continue;
+      }
+      // second panel of the pair: both panels' L21 from this panel's trailing rows on
+      Split v{pair + LB * pitch, rows_pad_all - LB, 256, 1};
+      Split head{pair + LB * pitch, LB, 256, 1};
+      if (rows > LB) {
+        // side: the columns beyond the next block, A22[128:, 128:] -= V[128:] V[128:]^T, K = 256
+        if ((e = cudaEventRecord(cs->ev[1], s)) != cudaSuccess) return e;
+        if ((e = cudaStreamWaitEvent(cs->side, cs->ev[1], 0)) != cudaSuccess) return e;
+        Split rest{v.p + LB * pitch, rows_pad_all - 2 * LB, 256, 1};
+        float* C22 = W + (o + 2 * LB) * d + (o + 2 * LB);
+        const int cap = num_sms() - 24;
+        e = syrk_tc(rest, gseg, hseg, 3, 256, C22, d, rows - LB, -1.f, 1.f, cap, st, cs->side);
+        if (e == cudaErrorNotSupported)
+          e = gemm_tc(rest, rest, 3, gseg, hseg, 256, C22, d, 0, rows - LB, rows - LB, -1.f, 1.f,
+                      true, 1, st, cs->side);
+        if (e != cudaSuccess) return e;
+        if ((e = cudaEventRecord(cs->ev[2 + ((p >> 1) & 1)], cs->side)) != cudaSuccess) return e;
+      } else if ((e = cudaEventRecord(cs->ev[2 + ((p >> 1) & 1)], cs->side)) != cudaSuccess) {
+        return e;
+      }
+      // critical: the next column block with both panels (K = 256)
+      if ((e = gemm_tc(v, head, 3, gseg, hseg, 256, W + (o + LB) * d + (o + LB), d, 0, rows,
+                       rows < LB ? rows : LB, -1.f, 1.f, true, 1, st, s,
+                       rows > LB ? &next_a21 : nullptr)) != cudaSuccess)
+        return e;
+    }
+    // the side stream's last update precedes the inverse
+    if ((e = cudaEventRecord(cs->ev[2], cs->side)) != cudaSuccess) return e;
+    if ((e = cudaStreamWaitEvent(s, cs->ev[2], 0)) != cudaSuccess) return e;
+    return cholesky_inverse(L, Linv, d, T, sb, st, s);
+  }
   for (int p = 0; p < np; ++p) {
     const int64_t o = (int64_t)p * LB;
     if ((e = launch_pdl(k_chol_leaf, dim3(1), dim3(LEAF_THREADS), LB_SMEM, s, W, d, d, o, L, d,
@@ -1314,7 +1445,6 @@ static cudaError_t cholesky_tc_body(const float* F, int64_t d, int64_t ldf, floa
     if ((!cs || p == 0) &&
         (e = split(W + (o + LB) * d + o, d, 0, rows, LB, false, a21, s)) != cudaSuccess)
       return e;
-    const int aseg[3] = {0, 0, 128}, bseg[3] = {0, 128, 0};
     // the epilogue also writes the split of L21 for the trailing update
     const int rows_pad = (rows + 127) / 128 * 128;
     Split l21{sb[cs ? 2 + 2 * (p & 1) : 2], rows_pad, 128, 1};
@@ -1360,50 +1490,7 @@ static cudaError_t cholesky_tc_body(const float* F, int64_t d, int64_t ldf, floa
     if ((e = cudaEventRecord(cs->ev[2 + (np & 1)], cs->side)) != cudaSuccess) return e;
     if ((e = cudaStreamWaitEvent(s, cs->ev[2 + (np & 1)], 0)) != cudaSuccess) return e;
   }
-  if (!Linv) return cudaSuccess;
-  // inverse by recursive doubling over block size b = 128, 256, ...
-  for (int64_t b = LB; b < d; b *= 2) {
-    const int64_t full_pairs = d / (2 * b);
-    const int64_t o_last = full_pairs * 2 * b;
-    const int64_t rows_last = d - o_last - b;
-    for (int part = 0; part < 2; ++part) {
-      const int batch = (int)(part == 0 ? full_pairs : (rows_last > 0 ? 1 : 0));
-      if (batch == 0) continue;
-      const int64_t o = part == 0 ? 0 : o_last;
-      const int rows = (int)(part == 0 ? b : rows_last);
-      const int64_t zs = 2 * b * d + 2 * b;  // source stride between pairs
-      const int kb = (int)((b + 63) / 64 * 64);
-      const int kr = (rows + 63) / 64 * 64;
-      const int rp = (rows + 127) / 128 * 128;
-      const int bp = (int)((b + 127) / 128 * 128);
-      // T_z = L21_z M11_z : A' = split(L21) (rows x b), B' = split(M11^T) (b x b)
-      Split l21{sb[0], rp, kb, batch};
-      Split m11t{sb[1], bp, kb, batch};
-      if ((e = split(L + (o + b) * d + o, d, zs, rows, (int)b, false, l21, s)) != cudaSuccess)
-        return e;
-      if ((e = split(Linv + o * d + o, d, zs, (int)b, (int)b, true, m11t, s)) != cudaSuccess)
-        return e;
-      const int as1[3] = {0, 0, kb}, bs1[3] = {0, kb, 0};
-      // B' = M11^T is upper triangular: output column block c needs k >= c
-      if ((e = gemm_tc(l21, m11t, 3, as1, bs1, (int)b, T, b, (int64_t)rp * b, rows, (int)b, 1.f,
-                       0.f, false, batch, st, s, nullptr, TRI_K_FROM_COL)) != cudaSuccess)
-        return e;
-      // M21_z = -M22_z T_z : A' = split(M22) (rows x rows), B' = split(T^T) (b x rows)
-      Split m22{sb[2], rp, kr, batch};
-      Split tt{sb[3], bp, kr, batch};
-      if ((e = split(Linv + (o + b) * d + (o + b), d, zs, rows, rows, false, m22, s)) !=
-          cudaSuccess)
-        return e;
-      // B'[c][k] = T[k][c]: b output rows, `rows` output columns
-      if ((e = split(T, b, (int64_t)rp * b, (int)b, rows, true, tt, s)) != cudaSuccess) return e;
-      const int as2[3] = {0, 0, kr}, bs2[3] = {0, kr, 0};
-      // A' = M22 is lower triangular: output row block r needs k < r + 128
-      if ((e = gemm_tc(m22, tt, 3, as2, bs2, rows, Linv + (o + b) * d + o, d, zs, rows, (int)b,
-                       -1.f, 0.f, false, batch, st, s, nullptr, TRI_K_TO_ROW)) != cudaSuccess)
-        return e;
-    }
-  }
-  return cudaSuccess;
+  return cholesky_inverse(L, Linv, d, T, sb, st, s);
 }
 
 }  // namespace ffh

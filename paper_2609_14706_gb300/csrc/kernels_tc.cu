@@ -443,382 +443,6 @@ cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t
 }
 
 // ===========================================================================
-// streamed weighted Gram (one CTA per output tile, weights applied on the way)
-// ===========================================================================
-// When the lower-triangle tiles about fill the GPU (d about 4096: 136 tiles of 256 x 256
-// on 148 SMs), every CTA owns one tile over the whole sample range, so there are no
-// split-K partials and no reduction kernel: the epilogue writes the finished tile and its
-// mirror image.  The weighted operand diag(w) V is produced a chunk of samples ahead by
-// the CTAs' own staging warps, which are idle while the MMAs run: each CTA scales its
-// share of the chunk (global -> registers -> global, no shared-memory traffic) into a ring
-// of NSLOT chunk slots that stays in L2; per-slot counters (release / acquire at GPU scope)
-// say when a slot is complete (every CTA wrote its share) and when it may be rewritten
-// (every CTA's TMA has read it).  The A operand then comes from the ring by TMA, B from
-// V.  A cooperative launch guarantees that all CTAs are resident together; every wait is
-// bounded.
-namespace gs {
-constexpr int BM = 256, BN = 256, BK = 64, STAGES = 3;
-constexpr int BOX_BYTES = 64 * BK * 2;
-constexpr int A_BYTES = BM * BK * 2;
-constexpr int B_BYTES = BN * BK * 2;
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr uint32_t TMEM_COLS = 512;
-constexpr int THREADS = 384;
-constexpr int NSCALE = THREADS - 128;
-constexpr int CH = 1024;          // samples per ring chunk (the ring stays in L2)
-constexpr int CB = CH / BK;       // sample blocks per chunk
-constexpr int NSLOT = 3;          // ring slots
-constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
-}  // namespace gs
-
-struct GramStreamArgs {
-  const __nv_bfloat16* V;
-  int64_t ld, N, d, vpr;      // vpr: 16-byte vectors per ring row (pad8(d) / 8)
-  const float* w;             // weights (N entries)
-  __nv_bfloat16* ring;        // [NSLOT][CH][8 vpr]
-  unsigned* ready;            // [NSLOT]: CTAs that finished writing the slot, cumulative
-  unsigned* consumed;         // [NSLOT]: CTAs whose TMA finished reading the slot, cumulative
-  const int2* tiles;
-  int T, KB, NC;
-  float* C;
-  int64_t ldc;
-  float scale;
-  DevStatus* st;
-  unsigned long long budget_ns;
-};
-
-// Wait (one thread) until *cnt >= target; false on timeout, a local abort or a raised error.
-__device__ __forceinline__ bool wait_count(const unsigned* cnt, unsigned target,
-                                           volatile int* abort_flag, const DevStatus* st,
-                                           uint64_t budget_ns) {
-  if (ld_acquire_gpu(cnt) >= target) return true;
-  const uint64_t t0 = global_timer_ns();
-  while (true) {
-    if (ld_acquire_gpu(cnt) >= target) return true;
-    if (*abort_flag || halted(st)) return false;
-    if (global_timer_ns() - t0 > budget_ns) return false;
-    __nanosleep(100);
-  }
-}
-
-__global__ void __launch_bounds__(gs::THREADS, 1)
-    k_gram_stream(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
-                  const GramStreamArgs a) {
-  using namespace gs;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~uintptr_t(1023));
-  uint8_t* stages = smem;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
-  uint64_t* full = bars;
-  uint64_t* empty = bars + STAGES;
-  uint64_t* accf = bars + 2 * STAGES;
-  uint64_t* drain = accf + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  volatile int* skip_flag = abort_flag + 1;
-  volatile int* scaler_ok = abort_flag + 2;
-
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (threadIdx.x == 0) {
-    *skip_flag = halted(a.st) ? 1 : 0;
-    *abort_flag = 0;
-    *scaler_ok = 1;
-    for (int s = 0; s < STAGES; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
-    }
-    mbar_init(accf, 1);
-    mbar_init(drain, 1);
-    fence_mbar_init();
-  }
-  __syncthreads();
-  if (*skip_flag) return;  // an earlier step failed or the fit stopped (grid-uniform)
-  if (warp == 2) {
-    tmem_alloc(tmem_slot, TMEM_COLS);
-    tmem_relinquish();
-  }
-  if (warp == 0 && lane == 0) {
-    prefetch_tmap(&amap);
-    prefetch_tmap(&bmap);
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-  const uint64_t budget = a.budget_ns;
-  const int2 tt = a.tiles[blockIdx.x];
-  const unsigned T = (unsigned)a.T;
-
-  if (warp == 0) {
-    if (lane == 0) {
-      // ---------------- TMA producer: A from the ring, B from V ----------------
-      bool ok = true;
-      int kb = 0;
-      for (; kb < a.KB && ok; ++kb) {
-        const int c = kb / CB, slot = c % NSLOT;
-        if (kb % CB == 0) {
-          // every CTA has written its share of chunk c into the slot
-          if (!wait_count(a.ready + slot, T * (unsigned)(c / NSLOT + 1), abort_flag, a.st,
-                          budget)) {
-            ok = false;
-            break;
-          }
-          fence_proxy_async_global();
-        }
-        const int s = kb % STAGES;
-        const uint32_t ph = (kb / STAGES) & 1;
-        if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, budget)) {
-          ok = false;
-          break;
-        }
-        mbar_arrive_expect_tx(&full[s], STAGE_BYTES);
-        uint8_t* sa = stages + s * STAGE_BYTES;
-        uint8_t* sb = sa + A_BYTES;
-        const int yr = (kb % CB) * BK;
-#pragma unroll
-        for (int q = 0; q < BM / 64; ++q)
-          tma_load_3d(sa + q * BOX_BYTES, &amap, &full[s], tt.x * BM + q * 64, yr, slot);
-#pragma unroll
-        for (int q = 0; q < BN / 64; ++q)
-          tma_load_2d(sb + q * BOX_BYTES, &bmap, &full[s], tt.y * BN + q * 64, kb * BK);
-      }
-      if (!ok) {
-        *abort_flag = 1;
-        raise_error(a.st, FFH_ERR_TIMEOUT, 21);
-      }
-      const int first = kb > STAGES ? kb - STAGES : 0;
-      for (int j = first; j < kb; ++j) {
-        volatile int never = 0;
-        mbar_wait(&full[j % STAGES], (j / STAGES) & 1, &never, budget);
-      }
-    }
-  } else if (warp == 1) {
-    if (lane == 0) {
-      // ---------------- MMA issuer ----------------
-      constexpr uint32_t idesc = idesc_bf16_f32(128, BN, true, true);
-      bool ok = true;
-      for (int kb = 0; kb < a.KB; ++kb) {
-        const int s = kb % STAGES;
-        const uint32_t ph = (kb / STAGES) & 1;
-        if (!mbar_wait(&full[s], ph, abort_flag, budget)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        // the chunk's last block has landed: its ring slot is free as far as this CTA goes
-        if (kb % CB == CB - 1 || kb == a.KB - 1) red_release_gpu_add(a.consumed + (kb / CB) % NSLOT, 1u);
-        const uint32_t sa = smem_u32(stages + s * STAGE_BYTES);
-        const uint32_t sb = sa + A_BYTES;
-#pragma unroll
-        for (int k = 0; k < BK / 16; ++k) {
-          const uint64_t bd = sw128_desc(sb + k * 2048, BOX_BYTES, 1024);
-#pragma unroll
-          for (int hh = 0; hh < 2; ++hh) {
-            const uint64_t ad = sw128_desc(sa + hh * 2 * BOX_BYTES + k * 2048, BOX_BYTES, 1024);
-            mma_bf16(tmem + hh * BN, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
-          }
-        }
-        mma_commit(&empty[s]);
-      }
-      if (ok) mma_commit(accf);
-      if (!ok) {
-        *abort_flag = 1;
-        raise_error(a.st, FFH_ERR_TIMEOUT, 22);
-      }
-      mma_commit(drain);
-      volatile int never = 0;
-      mbar_wait(drain, 0, &never, budget);
-    }
-  } else if (warp >= 4) {
-    // ---------------- ring producer (scaled chunks), then the epilogue ----------------
-    const int t = threadIdx.x - 128;
-    const int64_t total = (int64_t)CH * a.vpr;
-    const int64_t v0 = total * blockIdx.x / a.T, v1 = total * (blockIdx.x + 1) / a.T;
-    bool ok = true;
-    for (int c = 0; c < a.NC; ++c) {
-      const int slot = c % NSLOT;
-      if (c >= NSLOT) {
-        // every CTA's TMA has read the chunk that used this slot before
-        if (t == 0)
-          *scaler_ok = wait_count(a.consumed + slot, T * (unsigned)(c / NSLOT), abort_flag,
-                                  a.st, budget) ? 1 : 0;
-        named_bar_sync(1, NSCALE);
-        if (!*scaler_ok) {
-          ok = false;
-          break;
-        }
-      }
-      __nv_bfloat16* dst = a.ring + (size_t)slot * CH * (size_t)(8 * a.vpr);
-      const int vpr = (int)a.vpr;
-      // UNROLL vectors per thread in flight at once: all loads first, then scale + store
-      constexpr int UNROLL = 8;
-      for (int vb = (int)v0 + t; vb < (int)v1; vb += UNROLL * NSCALE) {
-        uint4 x[UNROLL];
-        float wv[UNROLL];
-#pragma unroll
-        for (int u = 0; u < UNROLL; ++u) {
-          const int v = vb + u * NSCALE;
-          const int row = v / vpr, col = (v - row * vpr) * 8;
-          const int64_t grow = (int64_t)c * CH + row;
-          x[u] = make_uint4(0u, 0u, 0u, 0u);
-          wv[u] = 0.f;
-          if (v < (int)v1 && grow < a.N) {
-            x[u] = __ldg(reinterpret_cast<const uint4*>(a.V + grow * a.ld + col));
-            wv[u] = __ldg(a.w + grow);
-          }
-        }
-#pragma unroll
-        for (int u = 0; u < UNROLL; ++u) {
-          const int v = vb + u * NSCALE;
-          if (v < (int)v1) {
-            const int row = v / vpr, col = (v - row * vpr) * 8;
-            uint4 y = x[u];
-            y.x = scale_bf16x2(y.x, wv[u]);
-            y.y = scale_bf16x2(y.y, wv[u]);
-            y.z = scale_bf16x2(y.z, wv[u]);
-            y.w = scale_bf16x2(y.w, wv[u]);
-            *reinterpret_cast<uint4*>(dst + (size_t)row * (8 * vpr) + col) = y;
-          }
-        }
-      }
-      __threadfence();
-      fence_proxy_async_global();
-      named_bar_sync(1, NSCALE);
-      if (t == 0) red_release_gpu_add(a.ready + slot, 1u);
-    }
-    if (!ok) {
-      if (t == 0) {
-        *abort_flag = 1;
-        raise_error(a.st, FFH_ERR_TIMEOUT, 23);
-      }
-    } else {
-      // epilogue: C = scale * acc for this tile and its mirror image (diagonal tiles: the
-      // lower triangle, mirrored, so C is exactly symmetric)
-      const int wq = warp & 3, hh = (warp - 4) >> 2;
-      if (mbar_wait(accf, 0, abort_flag, budget)) {
-        tc_fence_after();
-        const int64_t i = (int64_t)tt.x * BM + hh * 128 + wq * 32 + lane;
-        const bool diag = tt.x == tt.y;
-#pragma unroll 1
-        for (int cb = 0; cb < BN / 16; ++cb) {
-          float v[16];
-          tmem_ld16(tmem + ((uint32_t)(wq * 32) << 16) + hh * BN + cb * 16, v);
-          if (i < a.d) {
-            const int64_t j0 = (int64_t)tt.y * BN + cb * 16;
-#pragma unroll
-            for (int j16 = 0; j16 < 16; ++j16) v[j16] *= a.scale;
-            // row i: four 16-byte stores where the whole run is in range and wanted
-            const bool whole = j0 + 16 <= a.d && (!diag || i >= j0 + 15) &&
-                               ((a.ldc | j0) & 3) == 0;
-            if (whole) {
-#pragma unroll
-              for (int q = 0; q < 4; ++q)
-                *reinterpret_cast<float4*>(a.C + i * a.ldc + j0 + 4 * q) =
-                    make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-            }
-#pragma unroll
-            for (int j16 = 0; j16 < 16; ++j16) {
-              const int64_t j = j0 + j16;
-              if (j < a.d && (!diag || i >= j)) {
-                if (!whole) a.C[i * a.ldc + j] = v[j16];
-                a.C[j * a.ldc + i] = v[j16];   // the mirror: lanes write consecutive i
-              }
-            }
-          }
-        }
-      } else if (t == 0) {
-        *abort_flag = 1;
-        raise_error(a.st, FFH_ERR_TIMEOUT, 24);
-      }
-    }
-  }
-
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 2) {
-    tc_fence_after();
-    tmem_dealloc(tmem, TMEM_COLS);
-  }
-}
-
-bool gram_stream_eligible(int64_t d, int sms) {
-  const int64_t nb = (d + gs::BM - 1) / gs::BM;
-  const int64_t T = nb * (nb + 1) / 2;
-  // one tile per CTA, all resident: worth it when the tiles about fill the GPU
-  return T <= sms && 10 * T >= 8 * (int64_t)sms;
-}
-
-size_t gram_stream_ring_bytes(int64_t d) {
-  return (size_t)gs::NSLOT * gs::CH * (size_t)((d + 7) / 8 * 8) * 2 + 256;
-}
-
-cudaError_t launch_gram_stream(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t ld,
-                               const float* w, float scale, float* C, int64_t ldc, void* ring,
-                               const int2* tiles_dev, int T, DevStatus* st, cudaStream_t s) {
-  using namespace gs;
-  const int64_t dp = (d + 7) / 8 * 8;
-  if (!w || ld % 8 || ld < dp || (reinterpret_cast<uintptr_t>(V) & 15) ||
-      (reinterpret_cast<uintptr_t>(ring) & 255))
-    return cudaErrorInvalidValue;
-  unsigned* counters = reinterpret_cast<unsigned*>(ring);
-  __nv_bfloat16* rbuf = reinterpret_cast<__nv_bfloat16*>(static_cast<char*>(ring) + 256);
-  CUtensorMap amap, bmap;
-  {
-    auto fn = encode_fn();
-    if (!fn) return cudaErrorInvalidValue;
-    cuuint64_t dims[3] = {(cuuint64_t)d, (cuuint64_t)CH, (cuuint64_t)NSLOT};
-    cuuint64_t strides[2] = {(cuuint64_t)dp * 2, (cuuint64_t)CH * dp * 2};
-    cuuint32_t box[3] = {64, (cuuint32_t)BK, 1};
-    cuuint32_t es[3] = {1, 1, 1};
-    if (fn(&amap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, rbuf, dims, strides, box, es,
-           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-      return cudaErrorInvalidValue;
-  }
-  if (!make_map_bf16(&bmap, V, (uint64_t)d, (uint64_t)N, (uint64_t)ld, 64, BK))
-    return cudaErrorInvalidValue;
-  static PerDeviceOnce attr;
-  cudaError_t e = smem_attr_once((const void*)k_gram_stream, SMEM_BYTES, attr);
-  if (e != cudaSuccess) return e;
-  // the counters start at zero (skipped, like the kernel, once the fit has stopped)
-  if ((e = launch_zero_f32(reinterpret_cast<float*>(counters), 2 * NSLOT, st, s)) != cudaSuccess)
-    return e;
-  GramStreamArgs g;
-  g.V = V;
-  g.ld = ld;
-  g.N = N;
-  g.d = d;
-  g.vpr = dp / 8;
-  g.w = w;
-  g.ring = rbuf;
-  g.ready = counters;
-  g.consumed = counters + NSLOT;
-  g.tiles = tiles_dev;
-  g.T = T;
-  g.KB = (int)((N + BK - 1) / BK);
-  g.NC = (int)((N + CH - 1) / CH);
-  g.C = C;
-  g.ldc = ldc;
-  g.scale = scale;
-  g.st = st;
-  g.budget_ns = kWaitBudgetNs;
-  cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3((unsigned)T);
-  cfg.blockDim = dim3(THREADS);
-  cfg.dynamicSmemBytes = SMEM_BYTES;
-  cfg.stream = s;
-  cudaLaunchAttribute at[1];
-  at[0].id = cudaLaunchAttributeCooperative;
-  at[0].val.cooperative = 1;
-  cfg.attrs = at;
-  cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, k_gram_stream, amap, bmap, g);
-  note_launches(1);
-  return e != cudaSuccess ? e : cudaGetLastError();
-}
-
-// ===========================================================================
 // fused quadratic form
 // ===========================================================================
 namespace qf {

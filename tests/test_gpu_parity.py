@@ -61,11 +61,12 @@ def test_weighted_gram_matches_oracle(N, d, weighted):
 
 
 @pytest.mark.parametrize("N,d", [(2048, 4096), (4097, 4096), (9000, 4096), (5000, 4000)])
-def test_streamed_weighted_gram_matches_oracle(N, d):
-    """Widths whose 256 x 256 lower-triangle tiles about fill the GPU (d about 4096) take the
-    streamed kernel: one CTA per tile, the weighted operand written a chunk of 2048 samples
-    ahead into a 3-slot ring (N = 9000 reuses the slots, 4097 and 5000 end in a partial
-    chunk, d = 4000 in a partial tile).  Same elementwise bound as the split-K kernel."""
+def test_weighted_gram_headline_width_matches_oracle(N, d):
+    """The headline width (d = 4096, and a partial last tile at 4000) with several sample
+    blocks and a ragged N: elementwise bound, determinism, exact symmetry, and the relative
+    Frobenius error, which is what the fit's accuracy depends on (a single fp32 TMEM
+    accumulator over very many samples stays inside the elementwise bound while losing an
+    order of magnitude here)."""
     wl = synth.WORKLOADS["llama7b_attn_4096"].with_(n=d, m=8)
     X, _ = synth.rank_one_samples(wl, seed=7, device="cuda", N=N)
     w = torch.rand(N, device="cuda", generator=torch.Generator("cuda").manual_seed(8)) * 3
@@ -74,13 +75,17 @@ def test_streamed_weighted_gram_matches_oracle(N, d):
         C = h.weighted_gram(X, w, scale)
         C2 = h.weighted_gram(X, w, scale)
     torch.cuda.synchronize()
-    assert torch.equal(C, C2), "the streamed Gram must be deterministic"
+    assert torch.equal(C, C2), "the weighted Gram must be deterministic"
     Vn, wn = oracle.as_f64(X), oracle.as_f64(w)
     ref = oracle.weighted_gram(Vn, wn, scale)
     Cn = oracle.as_f64(C)
     assert np.array_equal(Cn, Cn.T), "output must be exactly symmetric"
     bound = _bf16_gram_bound(Vn, wn, scale) + 1e-7 * np.abs(ref).max()
     assert np.all(np.abs(Cn - ref) <= bound), np.max(np.abs(Cn - ref) / bound)
+    # bf16 rounding of the weighted operand is unbiased (2^-9 relative per term, averaging
+    # out over N terms); 5e-4 leaves a wide margin over the ~1e-4 measured
+    rel = np.linalg.norm(Cn - ref) / np.linalg.norm(ref)
+    assert rel < 5e-4, rel
 
 
 def test_weighted_gram_f32_input():
@@ -122,7 +127,7 @@ def test_quad_form_matches_oracle(N, d):
 # ---------------------------------------------------------------------------
 @pytest.mark.parametrize("d,cond", [(64, 1e2), (129, 1e2), (200, 1e3), (257, 1e3), (512, 1e3),
                                     (1000, 1e4), (1001, 1e3), (1536, 1e3), (2304, 1e3),
-                                    (4096, 1e4)])
+                                    (4096, 1e4), (8200, 1e3)])
 def test_cholesky_matches_oracle(d, cond):
     """Cholesky factor L and inverse M = L^-1.  Unit roundoff of the arithmetic: bf16
     hi/lo split products on the tensor cores (u = 2^-16 per product, fp32 accumulation).
