@@ -22,8 +22,9 @@ def test_gram_traffic_summary_is_used_only_for_its_kernel_source(tmp_path, monke
     b = _bench()
     traffic = b.profiled_traffic("llama7b_attn_4096")
     if traffic is not None:
-        # the algorithmic minimum is the two bf16 operands (2 x 2.15 GB); more is re-reads
-        assert 4.0e9 < traffic < 1.0e10
+        # both operands are slices of the one bf16 V (2.15 GB), read at least once; the
+        # split-K partials add 0.36 GB; far more would be re-reads the summary must explain
+        assert 2.15e9 < traffic < 1.0e10
     # a summary whose hash is not the current source's is ignored
     fake = tmp_path / "profiles"
     fake.mkdir()

@@ -58,9 +58,12 @@ def test_static_gram_matches_allocating_entry_point_twice(lib):
         code, C, msg = _call_static(lib, V, w, scale)
         assert code == 0, msg
         torch.cuda.synchronize()
-        diff = np.abs(oracle.as_f64(C) - oracle.as_f64(ref))
-        assert np.all(diff <= _bound(V, w, scale) + 1e-7 * oracle.as_f64(ref).max())
         Cn = oracle.as_f64(C)
+        # against the oracle's weighted Gram directly, then against the allocating entry
+        exact = oracle.weighted_gram(oracle.as_f64(V), oracle.as_f64(w), scale)
+        bound = _bound(V, w, scale) + 1e-7 * np.abs(exact).max()
+        assert np.all(np.abs(Cn - exact) <= bound), np.max(np.abs(Cn - exact) / bound)
+        assert np.all(np.abs(Cn - oracle.as_f64(ref)) <= 2 * bound)
         assert np.array_equal(Cn, Cn.T)
 
 
@@ -70,7 +73,10 @@ def test_static_gram_unweighted_and_rejects_oversize(lib):
         ref = h.weighted_gram(X, None, 0.5)
     code, C, msg = _call_static(lib, X, None, 0.5)
     assert code == 0, msg
-    assert np.all(np.abs(oracle.as_f64(C) - oracle.as_f64(ref)) <= _bound(X, None, 0.5) + 1e-7)
+    Cn = oracle.as_f64(C)
+    exact = oracle.weighted_gram(oracle.as_f64(X), np.ones(X.shape[0]), 0.5)
+    assert np.all(np.abs(Cn - exact) <= _bound(X, None, 0.5) + 1e-7)
+    assert np.all(np.abs(Cn - oracle.as_f64(ref)) <= 2 * _bound(X, None, 0.5) + 1e-7)
     big = torch.empty(64, 8192, dtype=torch.bfloat16, device="cuda")
     code, _, msg = _call_static(lib, big, None, 1.0)
     assert code == 1 and "static scratch" in msg
