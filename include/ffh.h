@@ -91,7 +91,12 @@ typedef struct {
   int32_t fault;           /* FFH_FAULT_* (tests only) */
   int32_t profile;         /* 1: time the Gram, quadratic-form and Cholesky kernels with
                               CUDA events on the handle's stream (see ffh_get_timings) */
-  int32_t reserved[4];     /* must be zero */
+  int32_t no_graph;        /* 0 (default): ffh_fit with device-resident X and G records the
+                              work it enqueues as a CUDA graph the first time and replays it
+                              when the next fit on the handle has the same sizes, pointers,
+                              iters, tol and options (one launch instead of thousands);
+                              1: always enqueue kernel by kernel */
+  int32_t reserved[3];     /* must be zero */
 } ffh_options;
 
 /* Kernel timings accumulated over the calls made with opt.profile = 1. */

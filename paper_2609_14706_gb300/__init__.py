@@ -37,7 +37,7 @@ class ffh_options(ctypes.Structure):
                 ("variant", ctypes.c_int32), ("init_A", ctypes.c_void_p),
                 ("final_loglik", ctypes.c_int32), ("reserved0", ctypes.c_int32),
                 ("fault", ctypes.c_int32), ("profile", ctypes.c_int32),
-                ("reserved", ctypes.c_int32 * 4)]
+                ("no_graph", ctypes.c_int32), ("reserved", ctypes.c_int32 * 3)]
 
 
 class ffh_timings(ctypes.Structure):
@@ -134,7 +134,7 @@ class Handle:
     def __init__(self, dtype="bf16", damping: float = 0.0, variant: str = "flipflop",
                  init_A: Optional[torch.Tensor] = None, final_loglik: bool = False,
                  fault: int = 0, profile: bool = False,
-                 stream: Optional[torch.cuda.Stream] = None):
+                 stream: Optional[torch.cuda.Stream] = None, graph: bool = True):
         self._lib = load_library()
         self._keep = []
         self.opts = ffh_options()
@@ -148,6 +148,7 @@ class Handle:
         self.opts.final_loglik = int(bool(final_loglik))
         self.opts.fault = int(fault)
         self.opts.profile = int(bool(profile))
+        self.opts.no_graph = 0 if graph else 1
         self.stream = stream if stream is not None else torch.cuda.current_stream()
         self._h = ctypes.c_void_p()
         code = self._lib.ffh_create(ctypes.byref(self._h), ctypes.byref(self.opts),

@@ -56,6 +56,34 @@ struct ffh_ctx {
   };
   std::vector<Pending> pending;
   CholStreams chol_cs;  // look-ahead streams of the tensor-core Cholesky (created on first use)
+  // The last fit's enqueued work as a CUDA graph, replayed while the next fit matches `key`
+  // (everything the enqueued sequence and its kernel arguments depend on).
+  struct FitKey {
+    const void *X = nullptr, *G = nullptr;
+    int64_t N = 0, n = 0, m = 0;
+    int32_t iters = 0;
+    float tol = 0.f, damping = 0.f;
+    int32_t dtype = 0, variant = 0, init = 0, final_loglik = 0, profile = 0;
+    void* ws = nullptr;
+    size_t ws_bytes = 0;
+    bool operator==(const FitKey& o) const {
+      return X == o.X && G == o.G && N == o.N && n == o.n && m == o.m && iters == o.iters &&
+             tol == o.tol && damping == o.damping && dtype == o.dtype && variant == o.variant &&
+             init == o.init && final_loglik == o.final_loglik && profile == o.profile &&
+             ws == o.ws && ws_bytes == o.ws_bytes;
+    }
+  };
+  struct FitGraph {
+    FitKey key;
+    cudaGraphExec_t exec = nullptr;
+    bool failed = false;           // capture of `key` failed: enqueue it directly
+    long long launches = 0;        // kernels in the graph
+    std::vector<Pending> pending;  // profile intervals the graph records
+    std::vector<cudaEvent_t> events;
+  } fg;
+  cudaStream_t cap_stream = nullptr;  // private stream the fit is captured on
+  bool capturing = false;
+  std::vector<cudaEvent_t> cap_events;  // profile events created while capturing
 };
 
 namespace {
@@ -126,6 +154,13 @@ ffh_status ensure_ws(ffh_t h, size_t bytes) {
 enum { PROF_GRAM = 0, PROF_QFORM = 1, PROF_CHOL = 2 };
 
 cudaEvent_t next_event(ffh_t h) {
+  if (h->capturing) {
+    // owned by the graph being captured (recorded on every replay), not the reusable pool
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    h->cap_events.push_back(e);
+    return e;
+  }
   if (h->ev_used == h->ev_pool.size()) {
     cudaEvent_t e;
     if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
@@ -134,11 +169,20 @@ cudaEvent_t next_event(ffh_t h) {
   return h->ev_pool[h->ev_used++];
 }
 
+// Record a timing event; inside a capture it becomes a node of the graph, so every replay
+// records it (a plain record on a capturing stream only orders work).
+void prof_record(ffh_t h, cudaEvent_t e) {
+  if (h->capturing)
+    cudaEventRecordWithFlags(e, h->stream, cudaEventRecordExternal);
+  else
+    cudaEventRecord(e, h->stream);
+}
+
 // Start a timed region of `kind` on the handle's stream (no-op unless opt.profile).
 cudaEvent_t prof_begin(ffh_t h) {
   if (!h->opt.profile) return nullptr;
   cudaEvent_t e = next_event(h);
-  if (e) cudaEventRecord(e, h->stream);
+  if (e) prof_record(h, e);
   return e;
 }
 
@@ -148,7 +192,7 @@ void prof_end(ffh_t h, int kind, cudaEvent_t a, cudaEvent_t b_recorded = nullptr
   if (!b) {
     b = next_event(h);
     if (!b) return;
-    cudaEventRecord(b, h->stream);
+    prof_record(h, b);
   }
   h->pending.push_back({kind, a, b});
 }
@@ -166,6 +210,77 @@ void prof_resolve(ffh_t h) {
   }
   h->pending.clear();
   h->ev_used = 0;
+}
+
+void drop_fit_graph(ffh_t h) {
+  auto& g = h->fg;
+  if (g.exec) cudaGraphExecDestroy(g.exec);
+  for (cudaEvent_t e : g.events) cudaEventDestroy(e);
+  g = ffh_ctx::FitGraph{};
+}
+
+// Run `enqueue` (which puts a fit's kernels on h->stream) through a CUDA graph: replay the
+// handle's graph when `key` matches, else capture `enqueue` on a private stream, instantiate
+// and launch it.  A capture that fails for any reason is discarded and the work enqueued
+// directly (and `key` is not captured again).
+template <class F>
+ffh_status run_as_graph(ffh_t h, const ffh_ctx::FitKey& key, F&& enqueue) {
+  auto& g = h->fg;
+  if (g.key == key && (g.exec || g.failed)) {
+    if (g.failed) return enqueue();
+    CK(cudaGraphLaunch(g.exec, h->stream));
+    note_launches((int)g.launches);
+    h->pending.insert(h->pending.end(), g.pending.begin(), g.pending.end());
+    return FFH_OK;
+  }
+  drop_fit_graph(h);
+  g.key = key;
+  if (!h->cap_stream) CK(cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking));
+  if (!h->chol_cs.crit) {
+    const cudaError_t e = chol_streams_init(&h->chol_cs);
+    if (e != cudaSuccess) {
+      chol_streams_destroy(&h->chol_cs);
+      return fail(h, FFH_ERR_CUDA, "Cholesky streams: %s", cudaGetErrorString(e));
+    }
+  }
+  cudaStream_t user = h->stream;
+  CK(cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeThreadLocal));
+  h->stream = h->cap_stream;
+  h->capturing = true;
+  const size_t pend0 = h->pending.size();
+  const long long l0 = launches_so_far();
+  ffh_status es = enqueue();
+  cudaGraph_t graph = nullptr;
+  cudaError_t ce = cudaStreamEndCapture(h->cap_stream, &graph);
+  h->stream = user;
+  h->capturing = false;
+  const long long counted = launches_so_far() - l0;
+  std::vector<ffh_ctx::Pending> pend(h->pending.begin() + pend0, h->pending.end());
+  h->pending.resize(pend0);
+  std::vector<cudaEvent_t> evs;
+  evs.swap(h->cap_events);
+  cudaGraphExec_t exec = nullptr;
+  if (es == FFH_OK && ce == cudaSuccess && graph)
+    ce = cudaGraphInstantiateWithFlags(&exec, graph, 0);
+  if (graph) cudaGraphDestroy(graph);
+  // nothing ran during the capture: the launches counted there happen only when the graph does
+  note_launches(-(int)counted);
+  if (es != FFH_OK || ce != cudaSuccess || !exec) {
+    cudaGetLastError();
+    if (exec) cudaGraphExecDestroy(exec);
+    for (cudaEvent_t e : evs) cudaEventDestroy(e);
+    g.failed = true;
+    h->err.clear();
+    return enqueue();
+  }
+  g.exec = exec;
+  g.launches = counted;
+  g.pending = std::move(pend);
+  g.events = std::move(evs);
+  CK(cudaGraphLaunch(g.exec, h->stream));
+  note_launches((int)g.launches);
+  h->pending.insert(h->pending.end(), g.pending.begin(), g.pending.end());
+  return FFH_OK;
 }
 
 ffh_status read_status(ffh_t h, DevStatus* st_dev, DevStatus* copy = nullptr) {
@@ -242,6 +357,8 @@ ffh_status ffh_destroy(ffh_t h) {
     cudaFree(h->ws);
   }
   for (cudaEvent_t e : h->ev_pool) cudaEventDestroy(e);
+  drop_fit_graph(h);
+  if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
   chol_streams_destroy(&h->chol_cs);
   delete h;
   return FFH_OK;
@@ -261,7 +378,9 @@ ffh_status validate_opt(ffh_t h) {
     return fail(h, FFH_ERR_INVALID_ARG, "damping must be finite and >= 0");
   if (o.variant < FFH_FLIPFLOP || o.variant > FFH_MARGINAL)
     return fail(h, FFH_ERR_INVALID_ARG, "bad variant %d", o.variant);
-  if (o.reserved0 != 0) return fail(h, FFH_ERR_INVALID_ARG, "reserved option field must be zero");
+  if (o.reserved0 != 0 || o.reserved[0] || o.reserved[1] || o.reserved[2])
+    return fail(h, FFH_ERR_INVALID_ARG, "reserved option field must be zero");
+  if (o.no_graph != 0 && o.no_graph != 1) return fail(h, FFH_ERR_INVALID_ARG, "no_graph must be 0 or 1");
   return FFH_OK;
 }
 
@@ -434,13 +553,13 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
   Carve c(h->ws);
   layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &tn, &ln,
          &tm, &lm, &partial, &trb, &Ares, &Bres);
-  cudaStream_t s = h->stream;
-  // the small kernels of this fit test its status block (see launch_iter_end)
+  // the small kernels of this fit (the input staging included) test its status block (see
+  // launch_iter_end), so it is cleared first, on every call, before anything is staged
   GateScope gate(st);
-  CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
-  CK(cudaMemsetAsync(recs, 0, sizeof(IterRecord) * (iters + 2), s));
-  CK(cudaMemsetAsync(q, 0, sizeof(float) * Npad, s));
-  CK(cudaMemsetAsync(r, 0, sizeof(float) * Npad, s));
+  CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), h->stream));
+  CK(cudaMemsetAsync(recs, 0, sizeof(IterRecord) * (iters + 2), h->stream));
+  CK(cudaMemsetAsync(q, 0, sizeof(float) * Npad, h->stream));
+  CK(cudaMemsetAsync(r, 0, sizeof(float) * Npad, h->stream));
   GramTables gtn, gtm;
   {
     ffh_status es = setup_tables(h, N, n, &gtn, tn, ln);
@@ -458,11 +577,8 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
 
   float* A[2] = {A2, A2 + (size_t)n * n};
   float* B[2] = {B2, B2 + (size_t)m * m};
-  int cur = 0;
   if (init) {
-    CK(cudaMemcpyAsync(A[cur], h->opt.init_A, sizeof(float) * n * n, cudaMemcpyDefault, s));
-  } else {
-    CK(launch_fill_identity(A[cur], n, n, s));
+    CK(cudaMemcpyAsync(A[0], h->opt.init_A, sizeof(float) * n * n, cudaMemcpyDefault, h->stream));
   }
   const float lam = h->opt.damping;
   const int variant = h->opt.variant;
@@ -470,101 +586,132 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
   const float sB = frob ? (float)(1.0 / (double)N) : (float)(1.0 / ((double)N * (double)n));
   const float sA = frob ? (float)(1.0 / (double)N) : (float)(1.0 / ((double)N * (double)m));
   int t_done = 0;
+  // Input / Marginal: one pass, no alternating loop
+  const int loop_iters = (variant == FFH_INPUT || variant == FFH_MARGINAL) ? 0 : iters;
   std::vector<IterRecord> host_recs((size_t)std::max(iters, 1) + 2);
-  if (variant == FFH_INPUT || variant == FFH_MARGINAL) {
-    // Table 1: A = E[x x^T]; B = I (Input) or E[g g^T] (Marginal); then tr A = n
-    const float s1 = (float)(1.0 / (double)N);
-    es = gram(h, xs, N, n, nullptr, s1, A[cur], partial, gtn, st);
-    if (es) return es;
-    if (variant == FFH_MARGINAL) {
-      es = gram(h, gs, N, m, nullptr, s1, B[cur], partial, gtm, st);
+  // Everything from here to the result selection is enqueued by `enqueue`, directly or
+  // recorded once as a CUDA graph and replayed (run_as_graph); nothing in it waits for the
+  // host.
+  auto enqueue = [&]() -> ffh_status {
+    cudaStream_t s = h->stream;
+    int cur = 0;
+    ffh_status es = FFH_OK;
+    if (!init) CK(launch_fill_identity(A[cur], n, n, s));
+    if (variant == FFH_INPUT || variant == FFH_MARGINAL) {
+      // Table 1: A = E[x x^T]; B = I (Input) or E[g g^T] (Marginal); then tr A = n
+      const float s1 = (float)(1.0 / (double)N);
+      es = gram(h, xs, N, n, nullptr, s1, A[cur], partial, gtn, st);
       if (es) return es;
-    } else {
-      CK(launch_fill_identity(B[cur], m, m, s));
+      if (variant == FFH_MARGINAL) {
+        es = gram(h, gs, N, m, nullptr, s1, B[cur], partial, gtm, st);
+        if (es) return es;
+      } else {
+        CK(launch_fill_identity(B[cur], m, m, s));
+      }
+      CK(launch_damp(A[cur], n, n, lam, st, s));
+      CK(launch_damp(B[cur], m, m, lam, st, s));
+      CK(launch_normalize(A[cur], n, B[cur], m, recs + 1, st, s));
+      CK(launch_iter_end(st, recs + 1, 1, 0.f, cur, s));
     }
-    CK(launch_damp(A[cur], n, n, lam, st, s));
-    CK(launch_damp(B[cur], m, m, lam, st, s));
-    CK(launch_normalize(A[cur], n, B[cur], m, recs + 1, st, s));
-    CK(launch_iter_end(st, recs + 1, 1, 0.f, cur, s));
-    iters = 0;  // no alternating loop
-  }
-  for (int t = 1; t <= iters; ++t) {
-    IterRecord* R = recs + t;
-    const int nxt = cur ^ 1;
-    // ---- weights q_k = x_k^T A_{t-1}^-1 x_k  (Frobenius: x_k^T A_{t-1} x_k)
-    if (t == 1 && !init) {
-      CK(launch_rowsumsq(xs.raw, dtype, N, n, xs.ld_raw, q, s));
-    } else if (frob) {
-      es = chol(h, A[cur], n, L, nullptr, work, st, 0);
+    for (int t = 1; t <= loop_iters; ++t) {
+      IterRecord* R = recs + t;
+      const int nxt = cur ^ 1;
+      // ---- weights q_k = x_k^T A_{t-1}^-1 x_k  (Frobenius: x_k^T A_{t-1} x_k)
+      if (t == 1 && !init) {
+        CK(launch_rowsumsq(xs.raw, dtype, N, n, xs.ld_raw, q, s));
+      } else if (frob) {
+        es = chol(h, A[cur], n, L, nullptr, work, st, 0);
+        if (es) return es;
+        es = qform_fwd(h, xs, N, n, L, Mb, q, st);
+        if (es) return es;
+      } else {
+        es = chol(h, A[cur], n, L, Linv, work, st, 0);
+        if (es) return es;
+        CK(launch_copy_f64(&R->logdet_A_prev, &st->logdet, s));
+        if (t > 1) CK(launch_copy_f64(&recs[t - 1].logdet_A, &st->logdet, s));
+        es = qform(h, xs, N, n, Linv, Mb, q, st);
+        if (es) return es;
+        if (t > 1) CK(launch_dot(q, r, N, &recs[t - 1].sum_qr_A, trb + 8, s));
+      }
+      // ---- B-update
+      es = gram(h, gs, N, m, q, sB, B[nxt], partial, gtm, st);
       if (es) return es;
-      es = qform_fwd(h, xs, N, n, L, Mb, q, st);
+      if (frob) {
+        CK(launch_frob2(A[cur], n, trb + 4, trb + 8, s));
+        CK(launch_scale_by_inv(B[nxt], m, trb + 4, s));
+      }
+      CK(launch_damp(B[nxt], m, m, lam, st, s));
+      es = chol(h, B[nxt], m, L, frob ? nullptr : Linv, work, st,
+                (t == 1 && h->opt.fault == FFH_FAULT_BAD_PIVOT) ? FFH_FAULT_BAD_PIVOT : 0);
       if (es) return es;
-    } else {
-      es = chol(h, A[cur], n, L, Linv, work, st, 0);
+      CK(launch_copy_f64(&R->logdet_B, &st->logdet, s));
+      if (frob) {
+        es = qform_fwd(h, gs, N, m, L, Mb, r, st);
+      } else {
+        es = qform(h, gs, N, m, Linv, Mb, r, st);
+      }
       if (es) return es;
-      CK(launch_copy_f64(&R->logdet_A_prev, &st->logdet, s));
-      if (t > 1) CK(launch_copy_f64(&recs[t - 1].logdet_A, &st->logdet, s));
+      CK(launch_dot(q, r, N, &R->sum_qr_B, trb + 8, s));
+      // ---- A-update
+      es = gram(h, xs, N, n, r, sA, A[nxt], partial, gtn, st);
+      if (es) return es;
+      if (frob) {
+        CK(launch_frob2(B[nxt], m, trb + 5, trb + 8, s));
+        CK(launch_scale_by_inv(A[nxt], n, trb + 5, s));
+      }
+      CK(launch_damp(A[nxt], n, n, lam, st, s));
+      CK(launch_normalize(A[nxt], n, B[nxt], m, R, st, s));
+      // ---- convergence statistics and the on-device stopping test
+      CK(cudaMemsetAsync(&R->dA2, 0, sizeof(double) * 4, s));
+      CK(launch_trace(A[nxt], n, trb + 0, s));
+      CK(launch_trace(A[cur], n, trb + 1, s));
+      CK(launch_delta(A[nxt], A[cur], n, &R->dA2, &R->nA2, trb, trb + 8, s));
+      if (t > 1) {
+        CK(launch_trace(B[nxt], m, trb + 2, s));
+        CK(launch_trace(B[cur], m, trb + 3, s));
+        CK(launch_delta(B[nxt], B[cur], m, &R->dB2, &R->nB2, trb + 2, trb + 8, s));
+      }
+      CK(launch_iter_end(st, R, t, tol, nxt, s));
+      cur = nxt;
+    }
+    // the last completed iterate (the fit may have stopped before `iters`)
+    CK(launch_select_copy(st, A[0], A[1], Ares, n * n, s));
+    CK(launch_select_copy(st, B[0], B[1], Bres, m * m, s));
+    if (h->opt.final_loglik && variant == FFH_FLIPFLOP) {
+      CK(launch_resume(st, s));
+      es = chol(h, Ares, n, L, Linv, work, st, 0);
+      if (es) return es;
+      CK(launch_record_at_done(st, recs, offsetof(IterRecord, logdet_A), &st->logdet, s));
       es = qform(h, xs, N, n, Linv, Mb, q, st);
       if (es) return es;
-      if (t > 1) CK(launch_dot(q, r, N, &recs[t - 1].sum_qr_A, trb + 8, s));
+      CK(launch_dot(q, r, N, trb + 6, trb + 8, s));
+      CK(launch_record_at_done(st, recs, offsetof(IterRecord, sum_qr_A), trb + 6, s));
     }
-    // ---- B-update
-    es = gram(h, gs, N, m, q, sB, B[nxt], partial, gtm, st);
-    if (es) return es;
-    if (frob) {
-      CK(launch_frob2(A[cur], n, trb + 4, trb + 8, s));
-      CK(launch_scale_by_inv(B[nxt], m, trb + 4, s));
-    }
-    CK(launch_damp(B[nxt], m, m, lam, st, s));
-    es = chol(h, B[nxt], m, L, frob ? nullptr : Linv, work, st,
-              (t == 1 && h->opt.fault == FFH_FAULT_BAD_PIVOT) ? FFH_FAULT_BAD_PIVOT : 0);
-    if (es) return es;
-    CK(launch_copy_f64(&R->logdet_B, &st->logdet, s));
-    if (frob) {
-      es = qform_fwd(h, gs, N, m, L, Mb, r, st);
-    } else {
-      es = qform(h, gs, N, m, Linv, Mb, r, st);
-    }
-    if (es) return es;
-    CK(launch_dot(q, r, N, &R->sum_qr_B, trb + 8, s));
-    // ---- A-update
-    es = gram(h, xs, N, n, r, sA, A[nxt], partial, gtn, st);
-    if (es) return es;
-    if (frob) {
-      CK(launch_frob2(B[nxt], m, trb + 5, trb + 8, s));
-      CK(launch_scale_by_inv(A[nxt], n, trb + 5, s));
-    }
-    CK(launch_damp(A[nxt], n, n, lam, st, s));
-    CK(launch_normalize(A[nxt], n, B[nxt], m, R, st, s));
-    // ---- convergence statistics and the on-device stopping test
-    CK(cudaMemsetAsync(&R->dA2, 0, sizeof(double) * 4, s));
-    CK(launch_trace(A[nxt], n, trb + 0, s));
-    CK(launch_trace(A[cur], n, trb + 1, s));
-    CK(launch_delta(A[nxt], A[cur], n, &R->dA2, &R->nA2, trb, trb + 8, s));
-    if (t > 1) {
-      CK(launch_trace(B[nxt], m, trb + 2, s));
-      CK(launch_trace(B[cur], m, trb + 3, s));
-      CK(launch_delta(B[nxt], B[cur], m, &R->dB2, &R->nB2, trb + 2, trb + 8, s));
-    }
-    CK(launch_iter_end(st, R, t, tol, nxt, s));
-    cur = nxt;
-  }
-  // the last completed iterate (the fit may have stopped before `iters`)
-  CK(launch_select_copy(st, A[0], A[1], Ares, n * n, s));
-  CK(launch_select_copy(st, B[0], B[1], Bres, m * m, s));
-  if (h->opt.final_loglik && variant == FFH_FLIPFLOP) {
-    CK(launch_resume(st, s));
-    es = chol(h, Ares, n, L, Linv, work, st, 0);
-    if (es) return es;
-    CK(launch_record_at_done(st, recs, offsetof(IterRecord, logdet_A), &st->logdet, s));
-    es = qform(h, xs, N, n, Linv, Mb, q, st);
-    if (es) return es;
-    CK(launch_dot(q, r, N, trb + 6, trb + 8, s));
-    CK(launch_record_at_done(st, recs, offsetof(IterRecord, sum_qr_A), trb + 6, s));
-  }
+    return FFH_OK;
+  };
+  ffh_ctx::FitKey key;
+  key.X = X;
+  key.G = G;
+  key.N = N;
+  key.n = n;
+  key.m = m;
+  key.iters = iters;
+  key.tol = tol;
+  key.damping = h->opt.damping;
+  key.dtype = dtype;
+  key.variant = variant;
+  key.init = init ? 1 : 0;
+  key.final_loglik = h->opt.final_loglik;
+  key.profile = h->opt.profile;
+  key.ws = h->ws;
+  key.ws_bytes = h->ws_bytes;
+  const bool graphable = !h->opt.no_graph && h->opt.fault == FFH_FAULT_NONE && x_dev && g_dev;
+  es = graphable ? run_as_graph(h, key, enqueue) : enqueue();
+  if (es) return es;
+  cudaStream_t s = h->stream;
   CK(cudaMemcpyAsync(A_out, Ares, sizeof(float) * n * n, cudaMemcpyDefault, s));
   CK(cudaMemcpyAsync(B_out, Bres, sizeof(float) * m * m, cudaMemcpyDefault, s));
-  const int rec_count = std::max(iters, 1) + 2;
+  const int rec_count = std::max(loop_iters, 1) + 2;
   CK(cudaMemcpyAsync(host_recs.data(), recs, sizeof(IterRecord) * rec_count,
                      cudaMemcpyDeviceToHost, s));
   DevStatus hst;

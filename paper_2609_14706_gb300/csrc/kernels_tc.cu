@@ -433,7 +433,15 @@ cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t
   note_launches(1);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  if (after_main && (e = cudaEventRecord(after_main, s)) != cudaSuccess) return e;
+  if (after_main) {
+    // a timing event: inside a stream capture it must become a graph node of its own
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if ((e = cudaStreamIsCapturing(s, &cap)) != cudaSuccess) return e;
+    e = cap == cudaStreamCaptureStatusActive
+            ? cudaEventRecordWithFlags(after_main, s, cudaEventRecordExternal)
+            : cudaEventRecord(after_main, s);
+    if (e != cudaSuccess) return e;
+  }
   const int nb32 = (int)((d + 31) / 32);
   const int nbn = (int)((d + gram::BN - 1) / gram::BN);
   k_gram_reduce<<<dim3(nb32, nb32), dim3(32, 8), 0, s>>>(partial, lut_dev, nbn, plan.T, plan.S,

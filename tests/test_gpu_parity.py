@@ -245,6 +245,55 @@ def test_fit_tol_stops_early():
     assert abs(st["iters_done"] - ref.iters_done) <= 1
 
 
+@pytest.mark.parametrize("case,tol,final", [("tiny_64", 0.0, False), ("llama_small", 0.0, True),
+                                             ("tiny_64", 1e-4, True)])
+def test_fit_graph_replay_equals_direct_enqueue(case, tol, final):
+    """A repeated fit on the same buffers replays the CUDA graph recorded by the first one;
+    both must equal, bit for bit, the same fit enqueued kernel by kernel (no_graph), with
+    the same statistics (a tol-stopped fit included) and the same kernel-launch count."""
+    wl = FIT_CASES[case]
+    X, G = synth.rank_one_samples(wl, seed=0, device="cuda")
+    it = 40 if tol > 0 else wl.iters
+    runs = {}
+    for graph in (True, False):
+        with ffh.Handle(dtype=wl.dtype, final_loglik=final, graph=graph) as h:
+            out = []
+            for _ in range(3):
+                l0 = h.timings()["kernel_launches"]
+                A, B = h.fit(X, G, iters=it, tol=tol)
+                torch.cuda.synchronize()
+                st = h.stats()
+                out.append((A.cpu(), B.cpu(), st, h.timings()["kernel_launches"] - l0))
+            runs[graph] = out
+    A0, B0, st0, n0 = runs[False][0]
+    labels = [f"graph fit {k}" for k in range(3)] + [f"direct fit {k}" for k in (1, 2)]
+    for lab, (A, B, st, nl) in zip(labels, runs[True] + runs[False][1:]):
+        assert torch.equal(A, A0) and torch.equal(B, B0), (
+            lab, float((A - A0).norm() / A0.norm()), float((B - B0).norm() / B0.norm()))
+        assert st["iters_done"] == st0["iters_done"]
+        assert st["delta"] == st0["delta"] or (np.isnan(st["delta"]) and np.isnan(st0["delta"]))
+        if final:
+            assert np.array_equal(np.array(st["loglik"]), np.array(st0["loglik"]), equal_nan=True)
+        assert nl == n0
+
+
+def test_fit_graph_replay_keeps_profile_timings():
+    """Profiling survives the replay: each replayed fit adds its Gram, quadratic-form and
+    Cholesky intervals, as a directly enqueued fit does."""
+    wl = FIT_CASES["llama_small"]
+    X, G = synth.rank_one_samples(wl, seed=1, device="cuda")
+    for graph in (True, False):
+        with ffh.Handle(dtype="bf16", profile=True, graph=graph) as h:
+            h.fit(X, G, iters=3)
+            h.timings(reset=True)
+            for _ in range(2):
+                h.fit(X, G, iters=3)
+            tm = h.timings()
+        assert tm["gram_launches"] == 2 * 6 and tm["gram_ms"] > 0
+        assert tm["qform_launches"] == 2 * 5 and tm["qform_ms"] > 0
+        assert tm["chol_calls"] == 2 * 5 and tm["chol_ms"] > 0
+
+
 @pytest.mark.parametrize("case,tol", [("tiny_64", 1e-4), ("llama_small", 2e-3)])
 def test_stop_on_device_equals_fixed_count_fit(case, tol):
     """The stopping test runs on the device: the fit enqueues all `iters` iterations and
