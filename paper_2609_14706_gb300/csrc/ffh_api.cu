@@ -429,21 +429,21 @@ ffh_status gram(ffh_t h, const Staged& V, int64_t N, int64_t d, const float* w_p
 
 // q_k = ||L^T v_k||^2 = v_k^T F v_k for F = L L^T (the Frobenius variant's weights)
 ffh_status qform_fwd(ffh_t h, const Staged& V, int64_t N, int64_t d, const float* L,
-                     __nv_bfloat16* Mb, float* q, DevStatus* st) {
+                     __nv_bfloat16* Mb, float* q, float* qpart, DevStatus* st) {
   const int64_t ldm = pad8(d);
   CK(launch_lowerT_to_bf16(L, d, d, Mb, ldm, h->stream));
   cudaEvent_t t0 = prof_begin(h);
-  CK(launch_qform_tc(V.bf, N, d, V.ld_bf, Mb, ldm, q, st, h->stream, true));
+  CK(launch_qform_tc(V.bf, N, d, V.ld_bf, Mb, ldm, q, qpart, st, h->stream, true));
   prof_end(h, PROF_QFORM, t0);
   return FFH_OK;
 }
 
 ffh_status qform(ffh_t h, const Staged& V, int64_t N, int64_t d, const float* Linv,
-                 __nv_bfloat16* Mb, float* q, DevStatus* st) {
+                 __nv_bfloat16* Mb, float* q, float* qpart, DevStatus* st) {
   const int64_t ldm = pad8(d);
   CK(launch_lower_to_bf16(Linv, d, d, Mb, ldm, h->stream));
   cudaEvent_t t0 = prof_begin(h);
-  CK(launch_qform_tc(V.bf, N, d, V.ld_bf, Mb, ldm, q, st, h->stream));
+  CK(launch_qform_tc(V.bf, N, d, V.ld_bf, Mb, ldm, q, qpart, st, h->stream));
   prof_end(h, PROF_QFORM, t0);
   return FFH_OK;
 }
@@ -543,16 +543,19 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
   int2 *tn, *tm;
   int *ln, *lm;
   double* trb;
+  const size_t qpart_floats = std::max(qform_scratch_floats(N, n), qform_scratch_floats(N, m));
   {
     Carve c(nullptr);
     layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &tn,
            &ln, &tm, &lm, &partial, &trb, &Ares, &Bres);
+    c.take<float>(qpart_floats);
     ffh_status es = ensure_ws(h, c.off + 1024);
     if (es) return es;
   }
   Carve c(h->ws);
   layout(c, &st, &recs, &Xb, &Gb, &stage, &q, &r, &A2, &B2, &L, &Linv, &Mb, &work, &tn, &ln,
          &tm, &lm, &partial, &trb, &Ares, &Bres);
+  float* qpart = c.take<float>(qpart_floats);
   // the small kernels of this fit (the input staging included) test its status block (see
   // launch_iter_end), so it is cleared first, on every call, before anything is staged
   GateScope gate(st);
@@ -622,14 +625,14 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
       } else if (frob) {
         es = chol(h, A[cur], n, L, nullptr, work, st, 0);
         if (es) return es;
-        es = qform_fwd(h, xs, N, n, L, Mb, q, st);
+        es = qform_fwd(h, xs, N, n, L, Mb, q, qpart, st);
         if (es) return es;
       } else {
         es = chol(h, A[cur], n, L, Linv, work, st, 0);
         if (es) return es;
         CK(launch_copy_f64(&R->logdet_A_prev, &st->logdet, s));
         if (t > 1) CK(launch_copy_f64(&recs[t - 1].logdet_A, &st->logdet, s));
-        es = qform(h, xs, N, n, Linv, Mb, q, st);
+        es = qform(h, xs, N, n, Linv, Mb, q, qpart, st);
         if (es) return es;
         if (t > 1) CK(launch_dot(q, r, N, &recs[t - 1].sum_qr_A, trb + 8, s));
       }
@@ -646,9 +649,9 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
       if (es) return es;
       CK(launch_copy_f64(&R->logdet_B, &st->logdet, s));
       if (frob) {
-        es = qform_fwd(h, gs, N, m, L, Mb, r, st);
+        es = qform_fwd(h, gs, N, m, L, Mb, r, qpart, st);
       } else {
-        es = qform(h, gs, N, m, Linv, Mb, r, st);
+        es = qform(h, gs, N, m, Linv, Mb, r, qpart, st);
       }
       if (es) return es;
       CK(launch_dot(q, r, N, &R->sum_qr_B, trb + 8, s));
@@ -682,7 +685,7 @@ extern "C" ffh_status ffh_fit(ffh_t h, const void* X, const void* G, int64_t N, 
       es = chol(h, Ares, n, L, Linv, work, st, 0);
       if (es) return es;
       CK(launch_record_at_done(st, recs, offsetof(IterRecord, logdet_A), &st->logdet, s));
-      es = qform(h, xs, N, n, Linv, Mb, q, st);
+      es = qform(h, xs, N, n, Linv, Mb, q, qpart, st);
       if (es) return es;
       CK(launch_dot(q, r, N, trb + 6, trb + 8, s));
       CK(launch_record_at_done(st, recs, offsetof(IterRecord, sum_qr_A), trb + 6, s));
@@ -1057,19 +1060,22 @@ extern "C" ffh_status ffh_quad_form(ffh_t h, const void* V, const float* Linv, i
   };
   DevStatus* st;
   __nv_bfloat16 *Vb, *Mb;
+  const size_t qpart_floats = qform_scratch_floats(N, d);
   {
     Carve c(nullptr);
     layout(c, &st, &Vb, &Mb);
+    c.take<float>(qpart_floats);
     ffh_status es = ensure_ws(h, c.off + 1024);
     if (es) return es;
   }
   Carve c(h->ws);
   layout(c, &st, &Vb, &Mb);
+  float* qpart = c.take<float>(qpart_floats);
   CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), h->stream));
   Staged vs_;
   ffh_status es = stage_input(h, V, true, N, d, Vb, nullptr, &vs_);
   if (es) return es;
-  es = qform(h, vs_, N, d, Linv, Mb, q_out, st);
+  es = qform(h, vs_, N, d, Linv, Mb, q_out, qpart, st);
   if (es) return es;
   return read_status(h, st);
 }
@@ -1254,14 +1260,17 @@ extern "C" ffh_status ffh_phi_tilde(ffh_t h, const void* X, const void* G, int64
   __nv_bfloat16 *Xb, *Gb, *Mb;
   float *q, *r, *L, *Linv, *work;
   double* acc;
+  const size_t qpart_floats = std::max(qform_scratch_floats(N, n), qform_scratch_floats(N, m));
   {
     Carve c(nullptr);
     layout(c, &st, &Xb, &Gb, &q, &r, &L, &Linv, &Mb, &work, &acc);
+    c.take<float>(qpart_floats);
     ffh_status es = ensure_ws(h, c.off + 1024);
     if (es) return es;
   }
   Carve c(h->ws);
   layout(c, &st, &Xb, &Gb, &q, &r, &L, &Linv, &Mb, &work, &acc);
+  float* qpart = c.take<float>(qpart_floats);
   cudaStream_t s = h->stream;
   CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
   Staged xs, gs;
@@ -1273,12 +1282,12 @@ extern "C" ffh_status ffh_phi_tilde(ffh_t h, const void* X, const void* G, int64
   es = chol(h, A, n, L, Linv, work, st, 0);
   if (es) return es;
   CK(cudaMemcpyAsync(&acc[1], &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
-  es = qform(h, xs, N, n, Linv, Mb, q, st);
+  es = qform(h, xs, N, n, Linv, Mb, q, qpart, st);
   if (es) return es;
   es = chol(h, B, m, L, Linv, work, st, 0);
   if (es) return es;
   CK(cudaMemcpyAsync(&acc[2], &st->logdet, sizeof(double), cudaMemcpyDeviceToDevice, s));
-  es = qform(h, gs, N, m, Linv, Mb, r, st);
+  es = qform(h, gs, N, m, Linv, Mb, r, qpart, st);
   if (es) return es;
   CK(launch_dot(q, r, N, &acc[0], acc + 4, s));
   double hacc[3];
@@ -1333,14 +1342,17 @@ extern "C" ffh_status ffh_partial_gram(ffh_t h, const void* U, const void* V, in
   float *w, *L, *Linv, *work, *partial, *Ptmp;
   int2* tiles;
   int* lut;
+  const size_t qpart_floats = qform_scratch_floats(N, du);
   {
     Carve c(nullptr);
     layout(c, &st, &Ub, &Vb, &w, &L, &Linv, &Mb, &work, &partial, &tiles, &lut, &Ptmp);
+    c.take<float>(qpart_floats);
     ffh_status es = ensure_ws(h, c.off + 1024);
     if (es) return es;
   }
   Carve c(h->ws);
   layout(c, &st, &Ub, &Vb, &w, &L, &Linv, &Mb, &work, &partial, &tiles, &lut, &Ptmp);
+  float* qpart = c.take<float>(qpart_floats);
   cudaStream_t s = h->stream;
   CK(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
   CK(cudaMemsetAsync(w, 0, sizeof(float) * Npad, s));
@@ -1353,7 +1365,7 @@ extern "C" ffh_status ffh_partial_gram(ffh_t h, const void* U, const void* V, in
   if (F) {
     es = chol(h, F, du, L, Linv, work, st, 0);
     if (es) return es;
-    es = qform(h, us, N, du, Linv, Mb, w, st);
+    es = qform(h, us, N, du, Linv, Mb, w, qpart, st);
     if (es) return es;
   } else {
     CK(launch_rowsumsq(us.raw, dtype, N, du, us.ld_raw, w, s));

@@ -178,10 +178,23 @@ cudaError_t launch_gram_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t
                            float* partial, int2* tiles_dev, int* tile_lut_dev,
                            const GramPlan& plan, DevStatus* st, int fault, cudaStream_t s,
                            cudaEvent_t after_main = nullptr);
-// q_k = ||M v_k||^2, V bf16 N x d (pitch ld), M bf16 d x d lower (pitch ldm)
+// CTAs that share one 128-sample row block of the quadratic form (each takes a snake-ordered
+// share of the 256-wide column blocks): 1 below 4 column blocks, 2 below 24, then 4, which
+// keeps the row blocks in flight within L2 at large d
+inline int qform_groups(int64_t d) {
+  const int64_t nc = (d + 255) / 256;
+  return nc >= 24 ? 4 : (nc >= 4 ? 2 : 1);
+}
+// fp32 scratch of the quadratic form over N samples of width d: the per-group partial sums
+// when more than two groups share a row block (added in a fixed order afterwards)
+inline size_t qform_scratch_floats(int64_t N, int64_t d) {
+  return qform_groups(d) > 2 ? (size_t)qform_groups(d) * (size_t)N : 0;
+}
+// q_k = ||M v_k||^2, V bf16 N x d (pitch ld), M bf16 d x d lower (pitch ldm); qpart: at
+// least qform_scratch_floats(N, d) floats (may be null when that is 0)
 cudaError_t launch_qform_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t ld,
-                            const __nv_bfloat16* M, int64_t ldm, float* q, DevStatus* st,
-                            cudaStream_t s, bool upper = false);
+                            const __nv_bfloat16* M, int64_t ldm, float* q, float* qpart,
+                            DevStatus* st, cudaStream_t s, bool upper = false);
 // fp32 -> bf16 of the transpose of a lower-triangular matrix (upper result, zeros below)
 cudaError_t launch_lowerT_to_bf16(const float* src, int64_t d, int64_t lds, __nv_bfloat16* dst,
                                   int64_t ldd, cudaStream_t s);

@@ -466,12 +466,22 @@ constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
 constexpr int THREADS = 256;
 }  // namespace qf
 
+// Group of column block c when G CTAs share a row block: the blocks are dealt out in a
+// snake (0, 1, .., G-1, G-1, .., 1, 0, 0, 1, ..), which balances the triangular K ranges
+// (block c costs c + 1 K-blocks of 256).
+__host__ __device__ inline int qf_group(int c, int G) {
+  const int p = c % (2 * G);
+  return p < G ? p : 2 * G - 1 - p;
+}
+
 struct QformArgs {
   float* q;
+  float* qpart;  // [G][N] per-group partial sums when G > 2
   int64_t N;
   int upper;  // M upper-triangular (column block c needs K >= 256 c) instead of lower
-  int G;     // column-block groups per row block (1 or 2): with 2, two CTAs share a row
-             // block (halving the L2 working set) and add their partial sums into q
+  int G;     // column-block groups per row block (qform_groups): G CTAs share a row block
+             // (dividing the L2 working set by G); with 2 they add their sums into q (two
+             // addends: order-independent), with more they write qpart, summed afterwards
   int RB;    // row blocks
   int NC;    // column blocks
   int KBd;   // 64-wide K blocks of d
@@ -535,7 +545,7 @@ __global__ void __launch_bounds__(qf::THREADS, 1)
       for (int u = blockIdx.x; u < a.RB * a.G && ok; u += gridDim.x) {
         const int rb = u / a.G, grp = u - rb * a.G;
         for (int c = 0; c < a.NC && ok; ++c) {
-          if (a.G == 2 && ((c + (c >> 1)) & 1) != grp) continue;
+          if (a.G > 1 && qf_group(c, a.G) != grp) continue;
           const int kb_lo = a.upper ? 4 * c : 0;
           const int kb_hi = a.upper ? a.KBd : min(a.KBd, 4 * (c + 1));
           for (int kb = kb_lo; kb < kb_hi; ++kb, ++it) {
@@ -570,7 +580,7 @@ __global__ void __launch_bounds__(qf::THREADS, 1)
       for (int u = blockIdx.x; u < a.RB * a.G && ok; u += gridDim.x) {
         const int grp = u % a.G;
         for (int c = 0; c < a.NC; ++c) {
-          if (a.G == 2 && ((c + (c >> 1)) & 1) != grp) continue;
+          if (a.G > 1 && qf_group(c, a.G) != grp) continue;
           const int buf = cc & 1;
           if (!mbar_wait(&acce[buf], ((cc >> 1) & 1) ^ 1, abort_flag, budget)) {
             ok = false;
@@ -620,7 +630,7 @@ __global__ void __launch_bounds__(qf::THREADS, 1)
       const int rb = u / a.G, grp = u - rb * a.G;
       float acc = 0.f;
       for (int c = 0; c < a.NC; ++c) {
-        if (a.G == 2 && ((c + (c >> 1)) & 1) != grp) continue;
+        if (a.G > 1 && qf_group(c, a.G) != grp) continue;
         const int buf = cc & 1;
         const uint32_t aph = (cc >> 1) & 1;
         ++cc;
@@ -643,7 +653,9 @@ __global__ void __launch_bounds__(qf::THREADS, 1)
       const int64_t row = (int64_t)rb * BM + wq * 32 + lane;
       // two groups: q was zeroed and receives exactly two addends (order-independent)
       if (row < a.N) {
-        if (a.G == 2)
+        if (a.G > 2)
+          a.qpart[(int64_t)grp * a.N + row] = acc;
+        else if (a.G == 2)
           atomicAdd(&a.q[row], acc);
         else
           a.q[row] = acc;
@@ -663,9 +675,21 @@ __global__ void __launch_bounds__(qf::THREADS, 1)
   }
 }
 
+// q_k = sum over the G groups of the partial sums, in group order (bit-reproducible)
+__global__ void k_qform_sum(const float* __restrict__ qpart, int G, int64_t N, float* q,
+                            const DevStatus* gate) {
+  if (gated_off(gate)) return;
+  for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < N;
+       k += (int64_t)gridDim.x * blockDim.x) {
+    float acc = qpart[k];
+    for (int g = 1; g < G; ++g) acc += qpart[(int64_t)g * N + k];
+    q[k] = acc;
+  }
+}
+
 cudaError_t launch_qform_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_t ld,
-                            const __nv_bfloat16* M, int64_t ldm, float* q, DevStatus* st,
-                            cudaStream_t s, bool upper) {
+                            const __nv_bfloat16* M, int64_t ldm, float* q, float* qpart,
+                            DevStatus* st, cudaStream_t s, bool upper) {
   CUtensorMap vmap, mmap;
   if (!make_map_bf16(&vmap, V, (uint64_t)d, (uint64_t)N, (uint64_t)ld, qf::BK, qf::BM))
     return cudaErrorInvalidValue;
@@ -678,22 +702,29 @@ cudaError_t launch_qform_tc(const __nv_bfloat16* V, int64_t N, int64_t d, int64_
   }
   QformArgs a;
   a.q = q;
+  a.qpart = qpart;
   a.N = N;
   a.upper = upper ? 1 : 0;
   a.RB = (int)((N + qf::BM - 1) / qf::BM);
   a.NC = (int)((d + qf::BN - 1) / qf::BN);
-  a.G = a.NC >= 4 ? 2 : 1;
+  a.G = qform_groups(d);
+  if (a.G > 2 && !qpart) return cudaErrorInvalidValue;
   a.KBd = (int)((d + qf::BK - 1) / qf::BK);
   a.st = st;
   a.budget_ns = kWaitBudgetNs;
   if (a.G == 2) {
-    // two addends per entry: q starts at zero (skipped, like the kernel, once the fit
-    // has stopped, so the last completed pass's values stay)
+    // the two groups add into q
     cudaError_t e = launch_zero_f32(q, N, st, s);
     if (e != cudaSuccess) return e;
   }
   const int grid = std::min(a.RB * a.G, num_sms());
-  k_qform_tc<<<grid, qf::THREADS, qf::SMEM_BYTES, s>>>(vmap, mmap, a); note_launches(1);
+  k_qform_tc<<<grid, qf::THREADS, qf::SMEM_BYTES, s>>>(vmap, mmap, a);
+  note_launches(1);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess || a.G <= 2) return e;
+  const int64_t blocks = std::min<int64_t>((N + 255) / 256, (int64_t)num_sms() * 8);
+  k_qform_sum<<<(unsigned)blocks, 256, 0, s>>>(qpart, a.G, N, q, st);
+  note_launches(1);
   return cudaGetLastError();
 }
 

@@ -104,14 +104,19 @@ def test_weighted_gram_f32_input():
 # ---------------------------------------------------------------------------
 # quadratic form
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("N,d", [(1000, 64), (3000, 264), (1500, 512), (129, 1024)])
+@pytest.mark.parametrize("N,d", [(1000, 64), (3000, 264), (1500, 512), (129, 1024), (700, 6400)])
 def test_quad_form_matches_oracle(N, d):
+    """d = 6400 has 25 column blocks of 256: four CTAs share each row block and their partial
+    sums are added in a fixed order (the result must not depend on which CTA finishes first)."""
     wl = synth.WORKLOADS["llama7b_attn_4096"].with_(n=d, m=8)
     X, _ = synth.rank_one_samples(wl, seed=4, device="cuda", N=N)
     A = oracle.as_f64(synth.spd_matrix(d, seed=5, cond=1e3, dtype=torch.float64))
     Linv = oracle.tri_inverse(oracle.cholesky(A))
     with ffh.Handle(dtype="bf16") as h:
-        q = h.quad_form(X, torch.tensor(Linv, dtype=torch.float32, device="cuda"))
+        Lt = torch.tensor(Linv, dtype=torch.float32, device="cuda")
+        q = h.quad_form(X, Lt)
+        q2 = h.quad_form(X, Lt)
+    assert torch.equal(q, q2), "the quadratic form must be deterministic"
     Xn = oracle.as_f64(X)
     ref = oracle.inv_quad_forms_chol(oracle.cholesky(A), Xn)
     Lf = Linv.astype(np.float32).astype(np.float64)   # what the kernel is given
