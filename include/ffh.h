@@ -50,7 +50,7 @@ typedef enum {
   FFH_ERR_OOM = 4,         /* workspace allocation failed */
   FFH_ERR_CUDA = 5,        /* a CUDA runtime call failed */
   FFH_ERR_TIMEOUT = 6,     /* a bounded device-side wait expired; the kernel returned */
-  FFH_ERR_UNSUPPORTED = 7  /* no sm_100-family GPU, or an option this build lacks */
+  FFH_ERR_UNSUPPORTED = 7  /* no sm_100-family GPU, or an option this library version lacks */
 } ffh_status;
 
 typedef enum { FFH_BF16 = 0, FFH_F32 = 1 } ffh_dtype;

@@ -1,7 +1,7 @@
 #!/usr/bin/env python
 """Full-size parity of the CUDA FlipFlop fit against the fp64 oracle.
 
-The spec configurations are too large for an oracle fit inside the GPU test run
+The five benchmark configurations are too large for an oracle fit inside the GPU test run
 (the fp64 fit of the 14336 x 4096 layer takes hours of host time), so the comparison
 runs in two halves that share only the portable seeded inputs (``synth.portable``):
 
@@ -263,8 +263,8 @@ def main() -> int:
     p = argparse.ArgumentParser()
     p.add_argument("half", choices=["gpu", "oracle"])
     p.add_argument("--configs", default=",".join(ALL))
-    p.add_argument("--out", default=os.path.join(ROOT, "gpurun_out", "parity"))
-    p.add_argument("--gpu", default=os.path.join(ROOT, "gpurun_out", "parity"))
+    p.add_argument("--out", default=os.path.join(ROOT, "parity_out"))
+    p.add_argument("--gpu", default=os.path.join(ROOT, "parity_out"))
     p.add_argument("--cache", default=os.path.join(ROOT, "tests", ".oracle_cache"))
     p.add_argument("--oracle-tol", type=float, default=1e-12,
                    help="oracle stopping tolerance for the --tol-configs workloads")
