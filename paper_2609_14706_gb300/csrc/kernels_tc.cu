@@ -379,13 +379,23 @@ GramPlan gram_plan(int64_t N, int64_t d, int sms) {
       if ((int64_t)tj * gram::BN <= (int64_t)ti * gram::BM + gram::BM - 1) ++T;
   p.T = T;
   p.KB = (int)std::max<int64_t>(1, (N + gram::BK - 1) / gram::BK);
-  // choose the split count: fill the SMs with equal-size units (wave efficiency),
-  // at least 8 blocks of samples per unit, partial buffer at most ~2 GB
-  int best_s = 1;
+  // Split count.  (1) No unit sums more than kMaxUnitSamples samples into its fp32
+  // accumulator: the error of one tensor-core accumulator over many MMAs grows with their
+  // number (a fit's Kronecker error measured 1.6e-4 with 26K samples per accumulator and
+  // 1.8e-3 with 262K).  (2) Among the counts that allow, fill the SMs with equal-size units
+  // (wave efficiency), at least 16 blocks of samples per unit.  (3) The partial tiles stay
+  // within kMaxPartialBytes (then (1) gives way).
+  constexpr int64_t kMaxUnitSamples = 32768;
+  constexpr double kMaxPartialBytes = 8.0e9;
+  const double unit_bytes = (double)gram::BN * gram::BM * 4.0;
+  const int s_acc = (int)((p.KB + kMaxUnitSamples / gram::BK - 1) / (kMaxUnitSamples / gram::BK));
+  const int s_mem = std::max(1, (int)(kMaxPartialBytes / ((double)T * unit_bytes)));
+  const int s_min = std::max(1, std::min(s_acc, s_mem));
+  const int max_s = std::max(s_min, std::min(64, p.KB / 16));
+  int best_s = s_min;
   double best_eff = -1.0;
-  const int max_s = std::max(1, std::min(64, p.KB / 16));
-  for (int s = 1; s <= max_s; ++s) {
-    if ((double)T * s * gram::BN * gram::BM * 4.0 > 2.0e9 && s > 1) break;
+  for (int s = s_min; s <= max_s; ++s) {
+    if ((double)T * s * unit_bytes > kMaxPartialBytes && s > s_min) break;
     const int64_t units = (int64_t)T * s;
     const int64_t waves = (units + sms - 1) / sms;
     const double eff = (double)units / (double)(waves * sms);
